@@ -1,0 +1,123 @@
+"""fp64 CPU oracle of the DAS hot path (ctypes loader for das_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: the test suite, the smoke check and the benchmark's
+CPU-baseline leg may use it; the CUDA library never does.  It shares no code
+with the CUDA path; only the seeded input generator (package `synth`) feeds
+both.
+
+Functions (each follows the paper; see das_oracle.c):
+  attend_seq       Eqs. 2-3 for one sequence and layer, on given slabs
+  attention        Eqs. 2-3 over a whole depth-indexed cache (Eq. 4 depths)
+  greedy_accept    Sec. 3.4 acceptance
+  kv_append        Sec. 3.4 / App. B.1 commit
+All pinned by tests/test_oracle_pins.py (no function is left unpinned).
+"""
+import ctypes
+import os
+
+import numpy as np
+
+from .build import LIB, build
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        L = ctypes.CDLL(LIB)
+        i, d, p = ctypes.c_int, ctypes.c_double, ctypes.c_void_p
+        L.das_oracle_attend_seq.argtypes = [i, i, i, i, i, i, p, p, p, p, p, i, i, i, d, p, p, i, i]
+        L.das_oracle_attend_seq.restype = None
+        L.das_oracle_attention.argtypes = [p, p, i, i, i, i, i, i, i, i, i, p, p, i, p, p, p, i, d,
+                                           i, p, p, i]
+        L.das_oracle_attention.restype = i
+        L.das_oracle_greedy_accept.argtypes = [p, p, i, i, i, p, p, p]
+        L.das_oracle_greedy_accept.restype = None
+        L.das_oracle_kv_append.argtypes = [p, p, i, i, i, i, i, i, p, p, p, i, p, p]
+        L.das_oracle_kv_append.restype = None
+        _lib = L
+    return _lib
+
+
+def _threads():
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def _u16(a):
+    return np.ascontiguousarray(a, dtype=np.uint16)
+
+
+def attend_seq(q, k_pre, v_pre, k_blk, v_blk, block_len=None, prefix_range=None, use_block=True,
+               scale=None, heads=None):
+    """One sequence, one layer.  q [T][Hq][D], k_pre/v_pre [P][Hkv][D],
+    k_blk/v_blk [T][Hkv][D], all bf16 bits.  Returns out [T][Hq][D] and
+    lse [Hq][T] in float64."""
+    q, k_pre, v_pre, k_blk, v_blk = map(_u16, (q, k_pre, v_pre, k_blk, v_blk))
+    T, Hq, D = q.shape
+    P, Hkv = k_pre.shape[0], k_pre.shape[1]
+    lo, hi = (0, P) if prefix_range is None else prefix_range
+    h_lo, h_hi = (0, Hq) if heads is None else heads
+    out = np.zeros((T, Hq, D))
+    lse = np.full((Hq, T), -np.inf)
+    lib().das_oracle_attend_seq(P, T, T if block_len is None else block_len, Hq, Hkv, D,
+                                q.ctypes.data, k_pre.ctypes.data, v_pre.ctypes.data,
+                                k_blk.ctypes.data, v_blk.ctypes.data, lo, hi, int(use_block),
+                                1.0 / np.sqrt(D) if scale is None else float(scale),
+                                out.ctypes.data, lse.ctypes.data, h_lo, h_hi)
+    return out, lse
+
+
+def attention(K, V, layer, key_depth, value_depth, prefix_len, block_len, q, k_blk, v_blk,
+              scale=None, use_block=True, nthreads=None):
+    """Whole cache.  K, V bf16 bits [R][L][B][cap][Hkv][D]; q [B][T][Hq][D];
+    k_blk, v_blk [B][T][Hkv][D].  Returns out [B][T][Hq][D], lse [B][Hq][T]."""
+    K, V, q, k_blk, v_blk = map(_u16, (K, V, q, k_blk, v_blk))
+    R, L, B, cap, Hkv, D = K.shape
+    T, Hq = q.shape[1], q.shape[2]
+    pl = np.ascontiguousarray(prefix_len, dtype=np.int32)
+    bl = np.ascontiguousarray(block_len, dtype=np.int32)
+    out = np.zeros((B, T, Hq, D))
+    lse = np.full((B, Hq, T), -np.inf)
+    rc = lib().das_oracle_attention(K.ctypes.data, V.ctypes.data, R, L, B, cap, Hkv, D, layer,
+                                    key_depth, value_depth, pl.ctypes.data, bl.ctypes.data, T,
+                                    q.ctypes.data, k_blk.ctypes.data, v_blk.ctypes.data, Hq,
+                                    0.0 if scale is None else float(scale), int(use_block),
+                                    out.ctypes.data, lse.ctypes.data, nthreads or _threads())
+    if rc:
+        raise ValueError("oracle: arguments outside the definition")
+    return out, lse
+
+
+def greedy_accept(logits, draft):
+    """logits float32 [B][W][V], draft int32 [B][W] ->
+    (accepted [B], target_ids [B][W], next_token [B]) int32."""
+    lg = np.ascontiguousarray(logits, dtype=np.float32)
+    dr = np.ascontiguousarray(draft, dtype=np.int32)
+    B, W, Vv = lg.shape
+    acc = np.zeros(B, dtype=np.int32)
+    tid = np.zeros((B, W), dtype=np.int32)
+    nxt = np.zeros(B, dtype=np.int32)
+    lib().das_oracle_greedy_accept(lg.ctypes.data, dr.ctypes.data, B, W, Vv, acc.ctypes.data,
+                                   tid.ctypes.data, nxt.ctypes.data)
+    return acc, tid, nxt
+
+
+def kv_append(K, V, k_new, v_new, accepted, prefix_len):
+    """Returns (K', V', prefix_len', error_flag) without touching the inputs.
+    K, V [R][L][B][cap][Hkv][D]; k_new, v_new [R][L][B][W][Hkv][D] (bf16 bits)."""
+    K2, V2 = np.array(K, dtype=np.uint16, copy=True), np.array(V, dtype=np.uint16, copy=True)
+    kn, vn = _u16(k_new), _u16(v_new)
+    R, L, B, cap, Hkv, D = K2.shape
+    W = kn.shape[3]
+    acc = np.ascontiguousarray(accepted, dtype=np.int32)
+    pl = np.array(prefix_len, dtype=np.int32, copy=True)
+    flag = np.zeros(1, dtype=np.int32)
+    lib().das_oracle_kv_append(K2.ctypes.data, V2.ctypes.data, R, L, B, cap, Hkv, D,
+                               kn.ctypes.data, vn.ctypes.data, acc.ctypes.data, W, pl.ctypes.data,
+                               flag.ctypes.data)
+    return K2, V2, pl, int(flag[0])
