@@ -1,0 +1,471 @@
+"""Benchmark of the DAS-Wave hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+  draft   L Mature-V draft-attention calls (keys at depth r, values at R),
+  verify  L full-depth verify-attention calls (depth R) over w candidate rows,
+  accept  greedy acceptance over [B, w, vocab] fp32 logits,
+  append  commit of the accepted inputs' K/V at all R depths and L layers.
+`value` is the Mature-V draft attention's prefix-KV bandwidth (GB/s): the
+algorithmic bytes the draft calls must read (K at depth r plus V at depth R,
+sum_b P_b * Hkv * D * 2 bytes each, per layer) over their device time,
+measured with CUDA events on the launch stream.  Inputs are resident in HBM
+before the timed region; L2 is flushed (a 512 MiB write) before every timed
+step.  `e2e` repeats the draft phase through the public Python/C API with the
+step's inputs copied from pinned host memory and its outputs read back.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+    python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
+
+With N > 1 (torchrun) every rank runs an independent replica on its own GPU
+(the path has no exchange step); value = bytes of all ranks / max time.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "decode"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="das", choices=["das", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="override the workload's layer count (smaller profiling captures)")
+    return ap.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_traffic(workload):
+    """dram bytes per attention launch from the committed ncu summary, if the
+    kernel source has not changed since it was captured; else None."""
+    src = os.path.join(ROOT, "paper_2609_34538_gb300", "csrc", "das_attention.cu")
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    path = os.path.join(ROOT, "profiles", "attn_kernel_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    for line in open(path):
+        parts = line.split()
+        if len(parts) == 3 and parts[0] == workload and parts[1] == digest:
+            return float(parts[2])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        if not getattr(self, "lines", None):
+            return None
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def gpu_arm(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_34538_gb300 as das
+    from synth import device as sdev
+    from synth import workloads as wlm
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+    wl = wlm.WORKLOADS[args.workload]
+    if args.layers:
+        wl = wl.replace(layers=args.layers)
+    if wl.kind != "draft":
+        raise SystemExit("the benchmark step needs a draft workload (its verify pass is derived)")
+    R, L, B = wl.depths, wl.layers, wl.batch
+    W = wl.max_block            # verify width: the draft block's rows are the candidates
+    vocab = 32000
+    wlv = wl.replace(key_depth=R, value_depth=R, seed=wl.seed + 1)
+
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        K, V = sdev.build_cache(wl, key_depths={wl.key_depth, R}, value_depths={R}, device=dev)
+        cache = das.DepthKVCache(K, V)
+        P0 = torch.from_numpy(wl.prefix_lens()).to(dev)
+        pl = P0.clone()
+        bl = torch.from_numpy(wl.block_lens()).to(dev)
+        ws = das.new_workspace(cache, wl.q_heads, W, device=dev)
+        draft_in = [sdev.layer_inputs(wl, l, dev) for l in range(L)]
+        verify_in = [sdev.layer_inputs(wlv, l, dev) for l in range(L)]
+        outs = [(torch.empty_like(q), torch.empty((B, wl.q_heads, W), dtype=torch.float32,
+                                                  device=dev)) for q, _, _ in draft_in]
+        vouts = [(torch.empty_like(q), torch.empty((B, wl.q_heads, W), dtype=torch.float32,
+                                                   device=dev)) for q, _, _ in verify_in]
+        acc_wl = wl.replace(vocab=vocab)
+        a_star, draft_ids, logits = sdev.accept_tensors(acc_wl, dev)
+        accepted = torch.empty(B, dtype=torch.int32, device=dev)
+        target = torch.empty((B, W), dtype=torch.int32, device=dev)
+        nxt = torch.empty(B, dtype=torch.int32, device=dev)
+        kn, vn = sdev.build_staged(wl, W, device=dev)
+        flag = torch.zeros(1, dtype=torch.int32, device=dev)
+        flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+    stream.synchronize()
+
+    def draft_phase():
+        for l, (q, kb, vb) in enumerate(draft_in):
+            das.das_mature_v_attention(cache, l, wl.key_depth, wl.value_depth, pl, bl, q, kb, vb,
+                                       ws, out=outs[l][0], lse=outs[l][1], stream=stream)
+
+    def verify_phase():
+        for l, (q, kb, vb) in enumerate(verify_in):
+            das.das_verify_attention(cache, l, R, pl, bl, q, kb, vb, ws, out=vouts[l][0],
+                                     lse=vouts[l][1], stream=stream)
+
+    def commit_phase():
+        das.das_greedy_accept(logits, draft_ids, accepted, target, nxt, stream=stream)
+        das.das_kv_append(cache, kn, vn, accepted, pl, flag, stream=stream)
+
+    # one eager pass (library set-up), then CUDA graphs of the three phases
+    with torch.cuda.stream(stream):
+        pl.copy_(P0)
+        draft_phase(); verify_phase(); commit_phase()
+    stream.synchronize()
+    graphs = []
+    for fn in (draft_phase, verify_phase, commit_phase):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        graphs.append(g)
+
+    def step(ev):
+        with torch.cuda.stream(stream):
+            pl.copy_(P0)          # every step commits onto the same prefix
+            flush.fill_(1)        # evict L2 (129 MB) before the timed phases
+            ev[0].record(stream)
+            graphs[0].replay()
+            ev[1].record(stream)
+            graphs[1].replay()
+            ev[2].record(stream)
+            graphs[2].replay()
+            ev[3].record(stream)
+
+    mk = lambda: [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    for _ in range(args.warmup):
+        step(mk())
+    stream.synchronize()
+    evs = [mk() for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        t0 = time.perf_counter()
+        for e in evs:
+            step(e)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    if world > 1:
+        dist.barrier()
+    draft_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    verify_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    commit_ms = [e[2].elapsed_time(e[3]) for e in evs]
+    step_ms = [e[0].elapsed_time(e[3]) for e in evs]
+
+    # correctness of what was timed: planted acceptance, no device-side errors
+    if not (np.array_equal(accepted.cpu().numpy(), a_star) and int(flag.item()) == 0
+            and das.workspace_status(ws) == 0):
+        raise SystemExit("bench: device results failed their checks")
+
+    draft_bytes = wl.prefix_bytes_per_layer() * L
+    verify_bytes = wlv.prefix_bytes_per_layer() * L
+    draft_s = sum(draft_ms) / 1e3
+    totals = torch.tensor([draft_s, sum(step_ms) / 1e3], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(totals, op=dist.ReduceOp.MAX)
+    draft_s, step_s = totals.tolist()
+    K_steps = args.steps
+    gbs = world * draft_bytes * K_steps / draft_s / 1e9
+    tokens = int(wl.block_lens().sum())
+    peak, peak_kind = peaks()
+    per_launch_ms = statistics.mean(draft_ms) / L
+    achieved = wl.prefix_bytes_per_layer() / (per_launch_ms / 1e3) / 1e9
+    traffic = kernel_traffic(args.workload)
+
+    e2e = None if args.no_e2e else e2e_arm(args, wl, cache, pl, P0, bl, ws, stream, dev)
+    if e2e is not None and world > 1:
+        t = torch.tensor([e2e.pop("_seconds")], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e["value"] = world * draft_bytes * K_steps / t.item() / 1e9
+    elif e2e is not None:
+        e2e.pop("_seconds")
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, budget_s=12.0)
+
+    line = {
+        "metric": "Mature-V draft-attn prefix-KV GB/s (% of GB300 HBM peak); draft tokens/s",
+        "value": round(gbs, 1),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": K_steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(statistics.mean(step_ms), 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded depth-maturation law; no datasets or weights)",
+        "config": {
+            "workload": wl.name,
+            "batch": B, "layers": L, "q_heads": wl.q_heads, "kv_heads": wl.kv_heads,
+            "head_dim": wl.head_dim, "depths": R, "key_depth": wl.key_depth,
+            "value_depth": wl.value_depth, "prefix_len": list(wl.prefix), "block": list(wl.block),
+            "verify_width": W, "vocab": vocab, "seed": wl.seed,
+            "parallelism": "replicas" if world > 1 else "single GPU",
+            "l2": "flushed before every timed step (512 MiB write)",
+        },
+        "pct_of_hbm_peak": {"measured_copy_6663.9" if peak_kind == "measured" else "fallback":
+                            round(100 * gbs / world / peak, 1),
+                            "nominal_8000": round(100 * gbs / world / 8000.0, 1)},
+        "draft_tokens_per_s": round(world * tokens * K_steps / draft_s, 1),
+        "phases_ms": {"draft": round(statistics.mean(draft_ms), 4),
+                      "verify": round(statistics.mean(verify_ms), 4),
+                      "accept_append": round(statistics.mean(commit_ms), 4)},
+        "verify_gbs": round(verify_bytes * K_steps / (sum(verify_ms) / 1e3) / 1e9, 1),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "kernel": "attn_kernel (one Mature-V layer call)",
+                     "peak_source": f"{peak_kind} HBM copy bandwidth"},
+        "gpu_launches": K_steps * (2 * L * 2 + 2 + 2),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "clocks": clocks.summary(),
+        "wall_s": round(wall, 3),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def e2e_arm(args, wl, cache, pl, P0, bl, ws, stream, dev):
+    """The draft phase through the public API with host buffers: each step
+    copies its queries and block K/V from pinned host memory, runs the L layer
+    calls and reads the outputs back."""
+    import torch
+
+    import paper_2609_34538_gb300 as das
+    from synth import workloads as wlm
+
+    L, B, W = wl.layers, wl.batch, wl.max_block
+    host_in = []
+    for l in range(L):
+        q = wlm.gen_q(wl, l)
+        kb, vb = wlm.gen_block_kv(wl, l)
+        host_in.append([torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).pin_memory()
+                        for x in (q, kb, vb)])
+    host_out = [(torch.empty(tuple(h[0].shape), dtype=torch.bfloat16).pin_memory(),
+                 torch.empty((B, wl.q_heads, W), dtype=torch.float32).pin_memory())
+                for h in host_in]
+    dev_in = [[torch.empty(tuple(x.shape), dtype=x.dtype, device=dev) for x in h] for h in host_in]
+    dev_out = [(torch.empty(tuple(h[0].shape), dtype=torch.bfloat16, device=dev),
+                torch.empty((B, wl.q_heads, W), dtype=torch.float32, device=dev)) for h in host_in]
+    bi = sum(x.numel() * x.element_size() for h in host_in for x in h)
+    bo = sum(o.numel() * o.element_size() + s.numel() * s.element_size() for o, s in host_out)
+
+    def step():
+        with torch.cuda.stream(stream):
+            for l in range(L):
+                for d, h in zip(dev_in[l], host_in[l]):
+                    d.copy_(h, non_blocking=True)
+                q, kb, vb = dev_in[l]
+                das.das_mature_v_attention(cache, l, wl.key_depth, wl.value_depth, pl, bl, q, kb,
+                                           vb, ws, out=dev_out[l][0], lse=dev_out[l][1],
+                                           stream=stream)
+                host_out[l][0].copy_(dev_out[l][0], non_blocking=True)
+                host_out[l][1].copy_(dev_out[l][1], non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        pl.copy_(P0)
+    for _ in range(args.warmup):
+        step()
+    stream.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    secs = e0.elapsed_time(e1) / 1e3
+    draft_bytes = wl.prefix_bytes_per_layer() * L
+    return {"value": round(draft_bytes * args.steps / secs / 1e9, 1), "unit": "GB/s",
+            "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,
+            "note": "L2 not flushed between e2e steps", "_seconds": secs}
+
+
+# ----------------------------------------------------------------------------- CPU legs
+
+def oracle_sample(wl, heads):
+    """Host inputs of the draft phase restricted to the first `heads` kv heads:
+    a 2-slab cache (slab 1 = keys at depth r, slab 2 = values at depth R)."""
+    from synth import T_KCACHE, T_VCACHE, matured_block
+    from synth import workloads as wlm
+    sub = wl.replace(kv_heads=heads, q_heads=heads * wl.group)
+    P = sub.prefix_lens()
+    shape = (2, sub.layers, sub.batch, int(P.max()) if P.max() > 0 else 1, heads, sub.head_dim)
+    K = np.zeros(shape, dtype=np.uint16)
+    V = np.zeros(shape, dtype=np.uint16)
+    for l in range(sub.layers):
+        for b in range(sub.batch):
+            n = int(P[b])
+            K[0, l, b, :n] = matured_block(sub.seed, T_KCACHE, 0, sub.key_depth, sub.depths, l, b,
+                                           0, n, 0, heads, sub.head_dim)
+            V[1, l, b, :n] = matured_block(sub.seed, T_VCACHE, 1, sub.value_depth, sub.depths, l,
+                                           b, 0, n, 0, heads, sub.head_dim)
+    ins = []
+    for l in range(sub.layers):
+        kb, vb = wlm.gen_block_kv(sub, l)
+        ins.append((wlm.gen_q(sub, l), kb, vb))
+    return sub, K, V, P, sub.block_lens(), ins
+
+
+def time_oracle(sub, K, V, P, T, ins, budget_s, min_reps=1):
+    import oracle
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    reps, t0 = 0, time.perf_counter()
+    while reps < min_reps or time.perf_counter() - t0 < budget_s:
+        for l, (q, kb, vb) in enumerate(ins):
+            oracle.attention(K, V, l, 1, 2, P, T, q, kb, vb, nthreads=cores)
+        reps += 1
+    secs = time.perf_counter() - t0
+    nbytes = int(P.astype(np.int64).sum()) * sub.kv_heads * sub.head_dim * 4 * sub.layers * reps
+    return nbytes / secs / 1e9, secs, reps, cores
+
+
+def sample_heads(wl, target_s=12.0):
+    """kv heads of the draft phase that the oracle covers in about target_s."""
+    return max(1, min(wl.kv_heads, 4 if wl.max_prefix > 10000 else wl.kv_heads))
+
+
+def cpu_baseline(wl, budget_s=12.0):
+    heads = sample_heads(wl)
+    sub, K, V, P, T, ins = oracle_sample(wl, heads)
+    gbs, secs, reps, cores = time_oracle(sub, K, V, P, T, ins, budget_s)
+    return {"value": round(gbs, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+            "sample": f"draft phase (all {wl.layers} layers) restricted to kv heads 0..{heads - 1} "
+                      f"of {wl.kv_heads}, repeated {reps}x in {secs:.1f} s; fp64, threaded over "
+                      "(sequence, query head)"}
+
+
+def reference_arm(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from synth import workloads as wlm
+    wl = wlm.WORKLOADS[args.workload]
+    heads = sample_heads(wl)
+    sub, K, V, P, T, ins = oracle_sample(wl, heads)
+    for _ in range(args.warmup):
+        time_oracle(sub, K, V, P, T, ins[:1], 0.0)
+    per_step = []
+    for _ in range(args.steps):
+        gbs, secs, reps, cores = time_oracle(sub, K, V, P, T, ins, 0.0)
+        per_step.append(secs)
+    nbytes = int(P.astype(np.int64).sum()) * heads * wl.head_dim * 4 * wl.layers
+    value = nbytes * args.steps / sum(per_step) / 1e9
+    sample = (f"per step: the draft phase ({wl.layers} layers) on kv heads 0..{heads - 1} of "
+              f"{wl.kv_heads}; fp64 oracle threaded over (sequence, query head)")
+    line = {"impl": "reference", "metric": "Mature-V draft-attn prefix-KV GB/s (% of GB300 HBM "
+            "peak); draft tokens/s", "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * statistics.mean(per_step), 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "sample_kv_heads": heads},
+            "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        gpu_arm(args)
+
+
+if __name__ == "__main__":
+    main()

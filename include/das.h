@@ -1,0 +1,187 @@
+/*
+ * das.h -- C ABI of the GB300 (sm_103a) library for the data-parallel hot path
+ * of DAS-Wave decoding ("Shallow Queries, Mature Values: Depth-Asynchronous
+ * Self-Speculation for Looped Transformers").
+ *
+ * The library computes, on one GPU:
+ *   das_mature_v_attention  depth-asynchronous draft attention, Eqs. 2-3
+ *                           (Sec. 3.2), with explicit read depths (Eq. 4):
+ *                           Mature-V is (key_depth, value_depth) = (r, R);
+ *   das_verify_attention    the full-depth verify attention of Sec. 3.4
+ *                           (Eq. 7): the same with key and value depth equal;
+ *   das_greedy_accept       greedy acceptance of Sec. 3.4;
+ *   das_kv_append           the commit of Sec. 3.4 / App. B.1.
+ *
+ * Conventions shared by every entry point
+ *   - Every pointer argument marked "device" is device memory owned by the
+ *     caller; the library never allocates or frees device memory.  Host
+ *     pointers are read during the call only.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; 0 = legacy default
+ *     stream) and never synchronise the host.  Errors found on the host
+ *     (arguments) are returned before anything is launched and nothing is
+ *     written.  Errors found on the device are reported through flags
+ *     described at each call.
+ *   - bf16 tensors are IEEE bfloat16, row-major in the stated index order,
+ *     densely packed, with base addresses aligned to 16 bytes.
+ *   - Recurrent depths are numbered as in the paper: 1..R, R = full depth.
+ *     Depth d is stored in slab d-1 of the cache.
+ *   - Query head h reads kv head h / G, G = num_q_heads / kv_heads
+ *     (contiguous grouping; the paper does not fix one).
+ */
+#ifndef DAS_H
+#define DAS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DAS_OK = 0,
+    DAS_ERR_INVALID_ARG = 1, /* a null pointer, bad size, depth or alignment */
+    DAS_ERR_UNSUPPORTED = 2, /* a shape outside what the kernels implement  */
+    DAS_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required  */
+    DAS_ERR_CUDA = 4         /* a CUDA runtime call failed                  */
+} das_status;
+
+/*
+ * Depth-indexed KV cache of the verified prefix (Sec. 2: the cache holds
+ * K_C^{r,l} and V_C^{r,l} for every recurrent depth r and core layer l; only
+ * target-materialized positions are stored, App. B.1).
+ *   k, v   device bf16 [depths][layers][batch][capacity][kv_heads][head_dim]
+ * Slab (d, l, b) is contiguous, so the keys of one depth and the values of
+ * another stream independently.  Positions >= prefix_len[b] may hold anything.
+ */
+typedef struct {
+    void *k;
+    void *v;
+    int depths;   /* R, number of stored recurrent depths, 1..63        */
+    int layers;   /* core layers                                        */
+    int batch;    /* sequences                                          */
+    int capacity; /* positions per sequence                             */
+    int kv_heads; /* Hkv                                                */
+    int head_dim; /* D: 64 or 128                                       */
+} das_kv_cache;
+
+/*
+ * Bytes of device workspace that das_mature_v_attention and
+ * das_verify_attention need for this cache shape, num_q_heads and max_block
+ * on the current device.  Returns 0 for shapes the kernels do not support.
+ * The first 256 bytes of a workspace are a header; its first int32 is a
+ * status word that the kernels OR with 1 if an internal wait ran out (a bug
+ * guard; it stays set until the caller clears it).  Zero a new workspace
+ * once before its first use.
+ */
+size_t das_workspace_size(const das_kv_cache *cache, int num_q_heads, int max_block);
+
+/*
+ * Depth-asynchronous attention, Eqs. 2-3 (Sec. 3.2).  For each sequence b,
+ * query head h and block row i < block_len[b]:
+ *   keys   = [ K[key_depth][layer][b][j][h/G]   for j < prefix_len[b] ]
+ *            ++ [ k_blk[b][j][h/G] for j <= i ]      (causal mask M)
+ *   values = [ V[value_depth][layer][b][j][h/G] for j < prefix_len[b] ]
+ *            ++ [ v_blk[b][j][h/G] for j <= i ]
+ *   s_j = softmax_scale * <q[b][i][h], keys_j>,  one softmax over all j,
+ *   out[b][i][h] = sum_j softmax(s)_j values_j,
+ *   lse[b][h][i] = ln sum_j exp(s_j).
+ * Mature-V for a draft at depth r is (key_depth, value_depth) = (r, R);
+ * Aligned (r, r), Deep K (R, r) and Deep K/V (R, R) are the other policies
+ * of Eq. 4.  The block's own K/V (k_blk, v_blk) are produced by the current
+ * draft and are never written to the cache by this call (Sec. 3.2, 3.3).
+ *
+ *   cache          the depth-indexed cache (read only)
+ *   layer          core layer, 0 <= layer < cache->layers
+ *   key_depth      kappa, 1..cache->depths
+ *   value_depth    nu, 1..cache->depths
+ *   prefix_len     device int32 [batch]: verified prefix length per sequence,
+ *                  0..capacity
+ *   block_len      device int32 [batch]: draft rows per sequence, 0..max_block
+ *   max_block      rows allocated per sequence in q/k_blk/v_blk/out/lse;
+ *                  (num_q_heads / kv_heads) * max_block <= 64, max_block <= 64
+ *   q              device bf16 [batch][max_block][num_q_heads][head_dim]
+ *   k_blk, v_blk   device bf16 [batch][max_block][kv_heads][head_dim]
+ *   num_q_heads    Hq, a multiple of kv_heads
+ *   softmax_scale  scale of Eq. 2; <= 0 selects 1/sqrt(head_dim)
+ *   out            device bf16 [batch][max_block][num_q_heads][head_dim];
+ *                  rows i >= block_len[b] are written as 0
+ *   lse            device fp32 [batch][num_q_heads][max_block]; -inf for rows
+ *                  i >= block_len[b]
+ *   workspace      device scratch of at least das_workspace_size() bytes,
+ *                  aligned to 256 bytes; calls sharing a workspace must not
+ *                  overlap in time
+ * Device-side: prefix_len or block_len outside their ranges are clamped and
+ * bit 1 of the workspace status word is set.
+ */
+das_status das_mature_v_attention(const das_kv_cache *cache, int layer, int key_depth,
+                                  int value_depth, const int32_t *prefix_len,
+                                  const int32_t *block_len, int max_block, const void *q,
+                                  const void *k_blk, const void *v_blk, int num_q_heads,
+                                  float softmax_scale, void *out, float *lse, void *workspace,
+                                  size_t workspace_bytes, void *stream);
+
+/*
+ * Independent full-depth verify attention (Sec. 3.4, Eq. 7): the verifier
+ * input [x_t, y_1 .. y_{w-1}] is the block (block_len[b] = w rows), it
+ * attends to the verified prefix at one depth for keys and values alike
+ * (depth = R for the target's last recurrence; every depth d of the verify
+ * pass uses the same call) and to itself under the causal mask.  Arguments
+ * and results as das_mature_v_attention with key_depth = value_depth = depth.
+ */
+das_status das_verify_attention(const das_kv_cache *cache, int layer, int depth,
+                                const int32_t *prefix_len, const int32_t *block_len,
+                                int max_block, const void *q, const void *k_blk,
+                                const void *v_blk, int num_q_heads, float softmax_scale,
+                                void *out, float *lse, void *workspace, size_t workspace_bytes,
+                                void *stream);
+
+/*
+ * Greedy acceptance (Sec. 3.4).  logits[b][i] stands for the verifier's
+ * conditional p_{i+1} of proposal y_{i+1} = draft_ids[b][i]:
+ *   target_ids[b][i] = argmax_v logits[b][i][v]   (smallest index on ties;
+ *                      binary32 comparisons; NaN logits are out of contract)
+ *   accepted[b]      = number of leading i with draft_ids[b][i] == target_ids[b][i]
+ *   next_token[b]    = target_ids[b][accepted[b]] if accepted[b] < W (the target
+ *                      prediction emitted at the first mismatch), otherwise
+ *                      draft_ids[b][W-1] (every proposal accepted: no further
+ *                      conditional exists, and the last accepted token becomes
+ *                      the next anchor).
+ *   logits      device fp32 [B][W][vocab]
+ *   draft_ids   device int32 [B][W]
+ *   accepted    device int32 [B];  target_ids device int32 [B][W];
+ *   next_token  device int32 [B]
+ * Requires 1 <= W <= 1024, 1 <= vocab < 2^31.
+ */
+das_status das_greedy_accept(const float *logits, const int32_t *draft_ids, int B, int W,
+                             int vocab, int32_t *accepted, int32_t *target_ids,
+                             int32_t *next_token, void *stream);
+
+/*
+ * Commit (Sec. 3.4; App. B.1): the verifier consumed W inputs
+ * [x_t, y_1 .. y_{W-1}] and produced their K/V at every depth and layer.
+ * With accepted[b] = a proposals accepted, the first n = min(a + 1, W) inputs
+ * (the anchor and the accepted proposals that were verifier inputs) are
+ * materialized: their staged K/V are copied byte for byte to cache positions
+ * prefix_len[b] .. prefix_len[b] + n - 1 at every depth and layer, and
+ * prefix_len[b] += n.  Rejected candidates' K/V are discarded.
+ *   k_new, v_new  device bf16 [depths][layers][batch][W][kv_heads][head_dim]
+ *   accepted      device int32 [batch] (as written by das_greedy_accept)
+ *   prefix_len    device int32 [batch], updated in place
+ *   error_flag    device int32: set to 1 (never cleared) if a sequence would
+ *                 exceed the capacity; that sequence's cache and prefix_len
+ *                 are left untouched
+ * Requires 1 <= W <= capacity.
+ */
+das_status das_kv_append(const das_kv_cache *cache, const void *k_new, const void *v_new,
+                         const int32_t *accepted, int W, int32_t *prefix_len,
+                         int32_t *error_flag, void *stream);
+
+/* Static text for a status code. */
+const char *das_status_string(das_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DAS_H */

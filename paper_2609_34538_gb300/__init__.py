@@ -1,0 +1,221 @@
+"""Python binding of libdas.so, the GB300 library for the data-parallel hot path
+of DAS-Wave decoding ("Shallow Queries, Mature Values: Depth-Asynchronous
+Self-Speculation for Looped Transformers").
+
+Argument marshalling only: every computation runs in the library's CUDA
+kernels.  PyTorch provides device memory and streams.  The names match the C
+ABI in include/das.h:
+
+    das_workspace_size      bytes of scratch the attention calls need
+    das_mature_v_attention  Eqs. 2-3 with explicit read depths (Eq. 4)
+    das_verify_attention    full-depth verify attention (Sec. 3.4, Eq. 7)
+    das_greedy_accept       greedy acceptance (Sec. 3.4)
+    das_kv_append           commit of accepted K/V at every depth (App. B.1)
+
+If libdas.so is missing the import fails: there is no fallback.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdas.so")
+
+DAS_OK, DAS_ERR_INVALID_ARG, DAS_ERR_UNSUPPORTED, DAS_ERR_WORKSPACE, DAS_ERR_CUDA = range(5)
+
+
+class DasError(RuntimeError):
+    def __init__(self, code, what):
+        super().__init__(f"{what}: {status_string(code)} (status {code})")
+        self.code = code
+
+
+class das_kv_cache(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("depths", ctypes.c_int),
+                ("layers", ctypes.c_int), ("batch", ctypes.c_int), ("capacity", ctypes.c_int),
+                ("kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is not built: run `python -m paper_2609_34538_gb300.build` "
+                          "(needs nvcc with sm_103a support)")
+    lib = ctypes.CDLL(LIB_PATH)
+    i, p, f, sz = ctypes.c_int, ctypes.c_void_p, ctypes.c_float, ctypes.c_size_t
+    cp = ctypes.POINTER(das_kv_cache)
+    lib.das_workspace_size.argtypes = [cp, i, i]
+    lib.das_workspace_size.restype = sz
+    lib.das_mature_v_attention.argtypes = [cp, i, i, i, p, p, i, p, p, p, i, f, p, p, p, sz, p]
+    lib.das_mature_v_attention.restype = i
+    lib.das_verify_attention.argtypes = [cp, i, i, p, p, i, p, p, p, i, f, p, p, p, sz, p]
+    lib.das_verify_attention.restype = i
+    lib.das_greedy_accept.argtypes = [p, p, i, i, i, p, p, p, p]
+    lib.das_greedy_accept.restype = i
+    lib.das_kv_append.argtypes = [cp, p, p, p, i, p, p, p]
+    lib.das_kv_append.restype = i
+    lib.das_status_string.argtypes = [i]
+    lib.das_status_string.restype = ctypes.c_char_p
+    return lib
+
+
+LIB = _load()
+
+
+def status_string(code):
+    return LIB.das_status_string(int(code)).decode()
+
+
+def _check(code, what):
+    if code != DAS_OK:
+        raise DasError(code, what)
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+
+
+def _need(t, dtype, name, ndim=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got {tuple(t.shape)}")
+
+
+class DepthKVCache:
+    """A depth-indexed cache: k, v bf16 [depths][layers][batch][capacity][kv_heads][head_dim]."""
+
+    def __init__(self, k, v):
+        _need(k, torch.bfloat16, "k", 6)
+        _need(v, torch.bfloat16, "v", 6)
+        if k.shape != v.shape:
+            raise ValueError("k and v shapes differ")
+        self.k, self.v = k, v
+        R, L, B, cap, H, D = k.shape
+        self.desc = das_kv_cache(k.data_ptr(), v.data_ptr(), R, L, B, cap, H, D)
+
+    @classmethod
+    def empty(cls, depths, layers, batch, capacity, kv_heads, head_dim, device="cuda"):
+        shape = (depths, layers, batch, capacity, kv_heads, head_dim)
+        return cls(torch.empty(shape, dtype=torch.bfloat16, device=device),
+                   torch.empty(shape, dtype=torch.bfloat16, device=device))
+
+    @property
+    def shape(self):
+        return tuple(self.k.shape)
+
+
+def das_workspace_size(cache, num_q_heads, max_block):
+    return int(LIB.das_workspace_size(ctypes.byref(cache.desc), num_q_heads, max_block))
+
+
+def new_workspace(cache, num_q_heads, max_block, device=None):
+    """Zeroed workspace tensor (uint8) of the size the attention calls need."""
+    n = das_workspace_size(cache, num_q_heads, max_block)
+    if n == 0:
+        raise DasError(DAS_ERR_UNSUPPORTED, "das_workspace_size")
+    return torch.zeros(n, dtype=torch.uint8, device=device or cache.k.device)
+
+
+def workspace_status(workspace):
+    """The workspace status word (bit 0: an internal wait timed out; bit 1: a
+    prefix or block length was out of range and clamped).  Synchronises."""
+    return int(workspace[:4].view(torch.int32).item())
+
+
+def _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse, workspace):
+    _need(prefix_len, torch.int32, "prefix_len", 1)
+    _need(block_len, torch.int32, "block_len", 1)
+    _need(q, torch.bfloat16, "q", 4)
+    _need(k_blk, torch.bfloat16, "k_blk", 4)
+    _need(v_blk, torch.bfloat16, "v_blk", 4)
+    R, L, B, cap, H, D = cache.shape
+    Bq, T, Hq, Dq = q.shape
+    if Bq != B or Dq != D or prefix_len.numel() != B or block_len.numel() != B:
+        raise ValueError("q / length shapes do not match the cache")
+    if tuple(k_blk.shape) != (B, T, H, D) or tuple(v_blk.shape) != (B, T, H, D):
+        raise ValueError("k_blk / v_blk must be [batch][max_block][kv_heads][head_dim]")
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((B, Hq, T), dtype=torch.float32, device=q.device)
+    _need(out, torch.bfloat16, "out", 4)
+    _need(lse, torch.float32, "lse", 3)
+    if tuple(out.shape) != tuple(q.shape) or tuple(lse.shape) != (B, Hq, T):
+        raise ValueError("out must be like q and lse [batch][num_q_heads][max_block]")
+    _need(workspace, torch.uint8, "workspace", 1)
+    return T, Hq, out, lse
+
+
+def das_mature_v_attention(cache, layer, key_depth, value_depth, prefix_len, block_len, q, k_blk,
+                           v_blk, workspace, out=None, lse=None, softmax_scale=0.0, stream=None):
+    """Depth-asynchronous attention (Eqs. 2-3); returns (out, lse)."""
+    T, Hq, out, lse = _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse,
+                                      workspace)
+    _check(LIB.das_mature_v_attention(
+        ctypes.byref(cache.desc), layer, key_depth, value_depth, _ptr(prefix_len),
+        _ptr(block_len), T, _ptr(q), _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale),
+        _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(stream)),
+        "das_mature_v_attention")
+    return out, lse
+
+
+def das_verify_attention(cache, layer, depth, prefix_len, block_len, q, k_blk, v_blk, workspace,
+                         out=None, lse=None, softmax_scale=0.0, stream=None):
+    """Full-depth verify attention (Sec. 3.4); returns (out, lse)."""
+    T, Hq, out, lse = _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse,
+                                      workspace)
+    _check(LIB.das_verify_attention(
+        ctypes.byref(cache.desc), layer, depth, _ptr(prefix_len), _ptr(block_len), T, _ptr(q),
+        _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale), _ptr(out), _ptr(lse),
+        _ptr(workspace), workspace.numel(), _stream(stream)), "das_verify_attention")
+    return out, lse
+
+
+def das_greedy_accept(logits, draft_ids, accepted=None, target_ids=None, next_token=None,
+                      stream=None):
+    """Greedy acceptance (Sec. 3.4); returns (accepted, target_ids, next_token)."""
+    _need(logits, torch.float32, "logits", 3)
+    _need(draft_ids, torch.int32, "draft_ids", 2)
+    B, W, V = logits.shape
+    if tuple(draft_ids.shape) != (B, W):
+        raise ValueError("draft_ids must be [B][W]")
+    dev = logits.device
+    accepted = torch.empty(B, dtype=torch.int32, device=dev) if accepted is None else accepted
+    target_ids = torch.empty((B, W), dtype=torch.int32, device=dev) if target_ids is None else target_ids
+    next_token = torch.empty(B, dtype=torch.int32, device=dev) if next_token is None else next_token
+    _need(accepted, torch.int32, "accepted", 1)
+    _need(target_ids, torch.int32, "target_ids", 2)
+    _need(next_token, torch.int32, "next_token", 1)
+    _check(LIB.das_greedy_accept(_ptr(logits), _ptr(draft_ids), B, W, V, _ptr(accepted),
+                                 _ptr(target_ids), _ptr(next_token), _stream(stream)),
+           "das_greedy_accept")
+    return accepted, target_ids, next_token
+
+
+def das_kv_append(cache, k_new, v_new, accepted, prefix_len, error_flag, stream=None):
+    """Commit (App. B.1): copy min(accepted+1, W) staged positions per sequence
+    at every depth and layer; prefix_len grows in place."""
+    _need(k_new, torch.bfloat16, "k_new", 6)
+    _need(v_new, torch.bfloat16, "v_new", 6)
+    _need(accepted, torch.int32, "accepted", 1)
+    _need(prefix_len, torch.int32, "prefix_len", 1)
+    _need(error_flag, torch.int32, "error_flag")
+    R, L, B, cap, H, D = cache.shape
+    W = k_new.shape[3]
+    if tuple(k_new.shape) != (R, L, B, W, H, D) or k_new.shape != v_new.shape:
+        raise ValueError("k_new / v_new must be [depths][layers][batch][W][kv_heads][head_dim]")
+    _check(LIB.das_kv_append(ctypes.byref(cache.desc), _ptr(k_new), _ptr(v_new), _ptr(accepted),
+                             W, _ptr(prefix_len), _ptr(error_flag), _stream(stream)),
+           "das_kv_append")

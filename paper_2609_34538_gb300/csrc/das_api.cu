@@ -1,0 +1,201 @@
+// das_api.cu -- the library's C ABI (include/das.h): argument checks, TMA
+// tensor-map encoding and launches.  Nothing here allocates device memory.
+#include <math.h>
+#include <mutex>
+
+#include "das_internal.h"
+
+namespace das {
+namespace {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// bf16 tensor map over `rank` dims (innermost first) with a {64, 1, 64, 1..}
+// box and 128-byte swizzle: one box is 64 positions x 64 head_dim elements.
+bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t strides[4];
+    cuuint64_t s = 2;
+    for (int i = 0; i < rank - 1; ++i) {
+        s *= dims[i];
+        strides[i] = s;
+    }
+    cuuint32_t box[5] = {64, 1, 64, 1, 1};
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, base, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool cache_ok(const das_kv_cache *c) {
+    return c && c->k && c->v && c->depths >= 1 && c->depths <= 63 && c->layers >= 1 &&
+           c->batch >= 1 && c->capacity >= 1 && c->kv_heads >= 1 &&
+           (c->head_dim == 64 || c->head_dim == 128) && aligned16(c->k) && aligned16(c->v);
+}
+
+das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_depth,
+                     const int32_t *prefix_len, const int32_t *block_len, int max_block,
+                     const void *q, const void *k_blk, const void *v_blk, int num_q_heads,
+                     float softmax_scale, void *out, float *lse, void *workspace,
+                     size_t workspace_bytes, void *stream) {
+    if (!cache_ok(c)) {
+        if (c && c->head_dim != 64 && c->head_dim != 128 && c->k && c->v) return DAS_ERR_UNSUPPORTED;
+        return DAS_ERR_INVALID_ARG;
+    }
+    if (layer < 0 || layer >= c->layers || key_depth < 1 || key_depth > c->depths ||
+        value_depth < 1 || value_depth > c->depths || !prefix_len || !block_len || !q ||
+        !k_blk || !v_blk || !out || !lse || num_q_heads < 1 || max_block < 1 ||
+        num_q_heads % c->kv_heads != 0 || !aligned16(q) || !aligned16(k_blk) ||
+        !aligned16(v_blk) || !aligned16(out) || !isfinite(softmax_scale))
+        return DAS_ERR_INVALID_ARG;
+    const int G = num_q_heads / c->kv_heads;
+    if (max_block > kTileKeys || (long long)G * max_block > kMaxRows) return DAS_ERR_UNSUPPORTED;
+    if ((long long)c->capacity > (1ll << 31) / 2 || c->batch > (1 << 20))
+        return DAS_ERR_UNSUPPORTED;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DAS_ERR_CUDA;
+    const size_t need = attn_workspace_bytes(dev, c->batch, c->kv_heads, G * max_block, c->head_dim);
+    if (need == 0) return DAS_ERR_CUDA;
+    if (!workspace || workspace_bytes < need ||
+        (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+        return DAS_ERR_WORKSPACE;
+
+    const int D = c->head_dim;
+    CUtensorMap tk, tv, tkb, tvb;
+    const cuuint64_t cache_dims[5] = {(cuuint64_t)D, (cuuint64_t)c->kv_heads,
+                                      (cuuint64_t)c->capacity, (cuuint64_t)c->batch,
+                                      (cuuint64_t)c->depths * c->layers};
+    const cuuint64_t blk_dims[4] = {(cuuint64_t)D, (cuuint64_t)c->kv_heads, (cuuint64_t)max_block,
+                                    (cuuint64_t)c->batch};
+    if (!encode_bf16(&tk, c->k, 5, cache_dims) || !encode_bf16(&tv, c->v, 5, cache_dims) ||
+        !encode_bf16(&tkb, const_cast<void *>(k_blk), 4, blk_dims) ||
+        !encode_bf16(&tvb, const_cast<void *>(v_blk), 4, blk_dims))
+        return DAS_ERR_CUDA;
+
+    AttnParams p;
+    p.prefix_len = prefix_len;
+    p.block_len = block_len;
+    p.q = static_cast<const uint16_t *>(q);
+    p.out = static_cast<uint16_t *>(out);
+    p.lse = lse;
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    p.status = reinterpret_cast<int32_t *>(ws);
+    p.B = c->batch;
+    p.Hq = num_q_heads;
+    p.Hkv = c->kv_heads;
+    p.G = G;
+    p.max_block = max_block;
+    p.rows_max = G * max_block;
+    p.capacity = c->capacity;
+    p.key_slab = (key_depth - 1) * c->layers + layer;
+    p.value_slab = (value_depth - 1) * c->layers + layer;
+    const double scale = softmax_scale > 0.f ? (double)softmax_scale : 1.0 / sqrt((double)D);
+    p.scale_log2 = (float)(scale * 1.4426950408889634);
+    p.num_ctas = attn_grid_size(dev);
+    const size_t slots = (size_t)c->batch * c->kv_heads + (size_t)p.num_ctas;
+    size_t off = kWorkspaceHeader;
+    p.part_o = reinterpret_cast<float *>(ws + off);
+    off += slots * p.rows_max * D * sizeof(float);
+    off = (off + 255) & ~size_t(255);
+    p.part_lse = reinterpret_cast<float *>(ws + off);
+    return attn_launch(p, D, tk, tv, tkb, tvb, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAS_OK
+               : DAS_ERR_CUDA;
+}
+
+}  // namespace
+}  // namespace das
+
+extern "C" {
+
+size_t das_workspace_size(const das_kv_cache *cache, int num_q_heads, int max_block) {
+    if (!cache || cache->kv_heads < 1 || num_q_heads < 1 || num_q_heads % cache->kv_heads != 0 ||
+        max_block < 1 || (cache->head_dim != 64 && cache->head_dim != 128))
+        return 0;
+    const int G = num_q_heads / cache->kv_heads;
+    if (max_block > das::kTileKeys || (long long)G * max_block > das::kMaxRows) return 0;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    return das::attn_workspace_bytes(dev, cache->batch, cache->kv_heads, G * max_block,
+                                     cache->head_dim);
+}
+
+das_status das_mature_v_attention(const das_kv_cache *cache, int layer, int key_depth,
+                                  int value_depth, const int32_t *prefix_len,
+                                  const int32_t *block_len, int max_block, const void *q,
+                                  const void *k_blk, const void *v_blk, int num_q_heads,
+                                  float softmax_scale, void *out, float *lse, void *workspace,
+                                  size_t workspace_bytes, void *stream) {
+    return das::attention(cache, layer, key_depth, value_depth, prefix_len, block_len, max_block,
+                          q, k_blk, v_blk, num_q_heads, softmax_scale, out, lse, workspace,
+                          workspace_bytes, stream);
+}
+
+das_status das_verify_attention(const das_kv_cache *cache, int layer, int depth,
+                                const int32_t *prefix_len, const int32_t *block_len,
+                                int max_block, const void *q, const void *k_blk,
+                                const void *v_blk, int num_q_heads, float softmax_scale,
+                                void *out, float *lse, void *workspace, size_t workspace_bytes,
+                                void *stream) {
+    return das::attention(cache, layer, depth, depth, prefix_len, block_len, max_block, q, k_blk,
+                          v_blk, num_q_heads, softmax_scale, out, lse, workspace, workspace_bytes,
+                          stream);
+}
+
+das_status das_greedy_accept(const float *logits, const int32_t *draft_ids, int B, int W,
+                             int vocab, int32_t *accepted, int32_t *target_ids,
+                             int32_t *next_token, void *stream) {
+    if (!logits || !draft_ids || !accepted || !target_ids || !next_token || B < 0 || W < 1 ||
+        W > 1024 || vocab < 1 || (long long)B * W > 0x7fffffffLL)
+        return DAS_ERR_INVALID_ARG;
+    return das::accept_launch(logits, draft_ids, B, W, vocab, accepted, target_ids, next_token,
+                              static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAS_OK
+               : DAS_ERR_CUDA;
+}
+
+das_status das_kv_append(const das_kv_cache *cache, const void *k_new, const void *v_new,
+                         const int32_t *accepted, int W, int32_t *prefix_len,
+                         int32_t *error_flag, void *stream) {
+    if (!das::cache_ok(cache) || !k_new || !v_new || !accepted || !prefix_len || !error_flag ||
+        W < 1 || W > cache->capacity || !das::aligned16(k_new) || !das::aligned16(v_new))
+        return DAS_ERR_INVALID_ARG;
+    return das::append_launch(*cache, k_new, v_new, accepted, W, prefix_len, error_flag,
+                              static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAS_OK
+               : DAS_ERR_CUDA;
+}
+
+const char *das_status_string(das_status s) {
+    switch (s) {
+        case DAS_OK: return "ok";
+        case DAS_ERR_INVALID_ARG: return "invalid argument";
+        case DAS_ERR_UNSUPPORTED: return "unsupported shape";
+        case DAS_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        case DAS_ERR_CUDA: return "CUDA runtime error";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,59 @@
+// das_internal.h -- declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "das.h"
+
+namespace das {
+
+// Work unit of the attention kernels: 64 key positions of one (sequence, kv
+// head).  Every (sequence, kv head) pair owns ceil(P/64) prefix tiles plus one
+// tile for the draft block's own keys.
+constexpr int kTileKeys = 64;
+constexpr int kMaxRows = 64;          // G * max_block handled by one pair
+constexpr int kConsumerWarps = 4;
+constexpr int kAttnThreads = kConsumerWarps * 32;
+constexpr int kCtasPerSm = 2;
+constexpr size_t kWorkspaceHeader = 256;
+
+// Bits of the workspace status word.
+constexpr int kStatusWaitTimeout = 1;
+constexpr int kStatusClamped = 2;
+
+struct AttnParams {
+    const int32_t *prefix_len;
+    const int32_t *block_len;
+    const uint16_t *q;  // bf16 [B][max_block][Hq][D]
+    uint16_t *out;      // bf16 [B][max_block][Hq][D]
+    float *lse;         // [B][Hq][max_block]
+    float *part_o;      // [slots][rows_max][D]
+    float *part_lse;    // [slots][rows_max]
+    int32_t *status;
+    int B, Hq, Hkv, G, max_block, rows_max, capacity;
+    int key_slab, value_slab;  // (depth - 1) * layers + layer
+    float scale_log2;          // softmax scale * log2(e)
+    int num_ctas;
+};
+
+// Number of CTAs the attention kernel launches on `device` (a persistent grid).
+int attn_grid_size(int device);
+size_t attn_workspace_bytes(int device, int batch, int kv_heads, int rows_max, int head_dim);
+
+// Launch the split-K attention kernel and its merge on `stream`.
+cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
+                        const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
+                        const CUtensorMap &tm_vb, cudaStream_t stream);
+
+cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
+                          int32_t *accepted, int32_t *target_ids, int32_t *next_token,
+                          cudaStream_t stream);
+
+cudaError_t append_launch(const das_kv_cache &c, const void *k_new, const void *v_new,
+                          const int32_t *accepted, int W, int32_t *prefix_len,
+                          int32_t *error_flag, cudaStream_t stream);
+
+}  // namespace das

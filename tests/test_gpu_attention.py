@@ -1,0 +1,147 @@
+"""Parity of das_mature_v_attention / das_verify_attention with the fp64
+oracle on seeded inputs, over shapes that span several tiles, splits across
+CTAs, ragged tails and the degenerate cases of the method."""
+import numpy as np
+import pytest
+import torch
+
+from synth import workloads as wl_mod
+from tests.gpu_util import dev_bf16, dev_i32, run_small
+
+pytestmark = pytest.mark.gpu
+
+TINY = wl_mod.WORKLOADS["tiny"]
+
+
+def small(**kw):
+    base = dict(name="small", batch=1, layers=2, q_heads=2, kv_heads=2, head_dim=128, depths=8,
+                key_depth=2, value_depth=8, prefix=(100, 100), block=(4,))
+    base.update(kw)
+    return wl_mod.Workload(**base)
+
+
+def test_tiny_workload():
+    """B1 L1 H4/4 D64 P256 T4 R8, Mature-V (r, R) = (2, 8)."""
+    run_small(TINY)
+
+
+@pytest.mark.parametrize("P", [0, 1, 63, 64, 65, 200, 1000])
+def test_prefix_lengths(P):
+    run_small(small(prefix=(P, P)), layer=1)
+
+
+@pytest.mark.parametrize("G,T", [(1, 1), (1, 16), (4, 4), (4, 8), (4, 12), (4, 16), (8, 8),
+                                 (1, 64), (2, 32)])
+def test_rows_per_kv_head(G, T):
+    """1..4 m-tiles of 16 rows (keys split 4, 2 or 1 ways between warps)."""
+    run_small(small(q_heads=2 * G, kv_heads=2, prefix=(300, 300), block=(T,)))
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_head_dims(D):
+    run_small(small(head_dim=D, q_heads=8, kv_heads=2, prefix=(777, 777), block=(8,)))
+
+
+def test_ragged_batch_with_empty_rows():
+    """Mixed prefix and block lengths, including P = 0 and T = 0."""
+    wl = small(batch=6, q_heads=8, kv_heads=2, block=(16,), prefix=(0, 600))
+    run_small(wl, prefix=[0, 1, 600, 64, 333, 0], block=[16, 0, 3, 8, 1, 0])
+
+
+def test_split_across_many_ctas():
+    """More tiles than CTAs for one pair: hundreds of partials merged."""
+    run_small(small(batch=1, kv_heads=1, q_heads=4, prefix=(20000, 20000), block=(16,)))
+    run_small(small(batch=2, kv_heads=2, q_heads=8, prefix=(5000, 5000), block=(8,)))
+
+
+def test_sharp_softmax_scale():
+    """scale = 1 makes the softmax peaked (the default 1/sqrt(D) is nearly flat here)."""
+    run_small(small(q_heads=8, kv_heads=2, prefix=(500, 500), block=(8,)), scale=1.0)
+
+
+@pytest.mark.parametrize("kap,nu", [(2, 8), (2, 2), (8, 2), (8, 8), (5, 3)])
+def test_read_policies(kap, nu):
+    """Eq. 4: Mature-V (r,R), Aligned (r,r), Deep K (R,r), Deep K/V (R,R), any pair."""
+    run_small(small(q_heads=4, kv_heads=2, prefix=(150, 150), block=(8,)), key_depth=kap,
+              value_depth=nu)
+
+
+def test_verify_attention():
+    run_small(small(q_heads=8, kv_heads=2, prefix=(400, 400), block=(16,), key_depth=8),
+              key_depth=8, value_depth=8, verify=True)
+
+
+def test_positions_past_the_prefix_are_never_read():
+    """NaN beyond prefix_len / block_len (cache, block K/V, queries) leaves the result exact."""
+    wl = small(batch=3, q_heads=8, kv_heads=2, block=(16,), prefix=(0, 300))
+    run_small(wl, prefix=[70, 300, 5], block=[5, 16, 9], poison_tail=True)
+
+
+def test_rows_past_block_are_zero_and_status_clean():
+    import paper_2609_34538_gb300 as das
+    wl = small(batch=2, q_heads=4, kv_heads=2, block=(16,), prefix=(0, 200))
+    out, lse, ws = run_small(wl, prefix=[200, 10], block=[3, 7])
+    o = out.float().cpu().numpy()
+    l = lse.cpu().numpy()
+    assert np.all(o[0, 3:] == 0) and np.all(o[1, 7:] == 0)
+    assert np.all(np.isneginf(l[0, :, 3:])) and np.all(np.isneginf(l[1, :, 7:]))
+    assert das.workspace_status(ws) == 0
+
+
+def test_out_of_range_lengths_are_clamped_and_flagged():
+    import paper_2609_34538_gb300 as das
+    wl = small(prefix=(50, 50), block=(4,))
+    cap = wl.capacity
+    from tests.gpu_util import dev_bf16 as up
+    K, V = wl_mod.gen_cache(wl, depths=[2, 8])
+    cache = das.DepthKVCache(up(K), up(V))
+    ws = das.new_workspace(cache, 2, 4)
+    q = up(wl_mod.gen_q(wl, 0))
+    kb, vb = map(up, wl_mod.gen_block_kv(wl, 0))
+    out1, l1 = das.das_mature_v_attention(cache, 0, 2, 8, dev_i32([cap + 100]), dev_i32([9]), q, kb,
+                                          vb, ws)
+    ws2 = das.new_workspace(cache, 2, 4)
+    out2, l2 = das.das_mature_v_attention(cache, 0, 2, 8, dev_i32([cap]), dev_i32([4]), q, kb, vb,
+                                          ws2)
+    torch.cuda.synchronize()
+    assert das.workspace_status(ws) == 2 and das.workspace_status(ws2) == 0
+    assert torch.equal(out1, out2) and torch.equal(l1, l2)
+
+
+def test_deterministic_and_graph_capturable():
+    import paper_2609_34538_gb300 as das
+    wl = small(batch=2, q_heads=8, kv_heads=2, prefix=(3000, 3000), block=(8,))
+    K, V = wl_mod.gen_cache(wl, depths=[2, 8])
+    cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+    ws = das.new_workspace(cache, 8, 8)
+    q = dev_bf16(wl_mod.gen_q(wl, 0))
+    kb, vb = map(dev_bf16, wl_mod.gen_block_kv(wl, 0))
+    pl, bl = dev_i32(wl.prefix_lens()), dev_i32(wl.block_lens())
+    o1, l1 = das.das_mature_v_attention(cache, 0, 2, 8, pl, bl, q, kb, vb, ws)
+    o2, l2 = das.das_mature_v_attention(cache, 0, 2, 8, pl, bl, q, kb, vb, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    o3, l3 = torch.zeros_like(o1), torch.zeros_like(l1)
+    s = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        das.das_mature_v_attention(cache, 0, 2, 8, pl, bl, q, kb, vb, ws, out=o3, lse=l3)
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o3) and torch.equal(l1, l3)
+
+
+def test_host_errors_raise():
+    import paper_2609_34538_gb300 as das
+    wl = small()
+    cache = das.DepthKVCache.empty(8, 2, 1, wl.capacity, 2, 128)
+    ws = das.new_workspace(cache, 2, 4)
+    q = torch.zeros((1, 4, 2, 128), dtype=torch.bfloat16, device="cuda")
+    kb = torch.zeros((1, 4, 2, 128), dtype=torch.bfloat16, device="cuda")
+    pl, bl = dev_i32([10]), dev_i32([4])
+    with pytest.raises(das.DasError) as e:
+        das.das_mature_v_attention(cache, 0, 9, 8, pl, bl, q, kb, kb, ws)
+    assert e.value.code == das.DAS_ERR_INVALID_ARG
+    with pytest.raises(das.DasError) as e:
+        das.das_mature_v_attention(cache, 0, 2, 8, pl, bl, q, kb, kb, ws[:100])
+    assert e.value.code == das.DAS_ERR_WORKSPACE

@@ -1,0 +1,116 @@
+"""Bit-exact parity of das_greedy_accept and das_kv_append with the oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from synth import workloads as wl_mod
+from tests.gpu_util import dev_bf16, dev_i32, host_bits
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_accept(logits, draft):
+    import paper_2609_34538_gb300 as das
+    acc, tid, nxt = das.das_greedy_accept(torch.from_numpy(logits).cuda(),
+                                          torch.from_numpy(draft).cuda())
+    torch.cuda.synchronize()
+    return acc.cpu().numpy(), tid.cpu().numpy(), nxt.cpu().numpy()
+
+
+def check_accept(logits, draft):
+    g = gpu_accept(np.ascontiguousarray(logits, np.float32), np.ascontiguousarray(draft, np.int32))
+    o = oracle.greedy_accept(logits, draft)
+    for a, b, name in zip(g, o, ["accepted", "target_ids", "next_token"]):
+        assert np.array_equal(a, b), name
+    return g
+
+
+def test_accept_verify_workload():
+    """[8, 16, 32000] fp32 logits ~ N(0, 4) with planted acceptance lengths."""
+    a_star, draft, logits = synth.accept_inputs(0, 8, 16, 32000)
+    acc, _, _ = check_accept(logits, draft)
+    assert np.array_equal(acc, a_star)
+
+
+@pytest.mark.parametrize("B,W,V", [(1, 1, 2), (3, 5, 1001), (2, 16, 7), (4, 32, 50257), (1, 3, 4)])
+def test_accept_shapes(B, W, V):
+    a_star, draft, logits = synth.accept_inputs(B * 100 + W, B, W, V)
+    check_accept(logits, draft)
+
+
+def test_accept_ties_and_infinities():
+    """Equal maxima go to the smallest index; rows of -inf give index 0."""
+    B, W, V = 3, 4, 4099
+    logits = np.zeros((B, W, V), dtype=np.float32)
+    logits[0, 0, [5, 9, 4000]] = 3.0
+    logits[0, 1, [4098, 4097]] = 1.0
+    logits[1, :, :] = -np.inf
+    logits[2, 2, 17] = np.inf
+    logits[2, 2, 18] = np.inf
+    draft = np.array([[5, 4097, 0, 0], [0, 0, 0, 1], [0, 0, 17, 3]], dtype=np.int32)
+    acc, tid, nxt = check_accept(logits, draft)
+    assert tid[0, 0] == 5 and tid[0, 1] == 4097 and np.all(tid[1] == 0) and tid[2, 2] == 17
+    assert list(acc) == [4, 3, 3]
+
+
+def _append_case(R, L, B, cap, H, D, W, pl, acc, seed):
+    import paper_2609_34538_gb300 as das
+    rng = np.random.default_rng(seed)
+    K = rng.integers(0, 65535, (R, L, B, cap, H, D), dtype=np.uint16)
+    V = rng.integers(0, 65535, (R, L, B, cap, H, D), dtype=np.uint16)
+    kn = rng.integers(0, 65535, (R, L, B, W, H, D), dtype=np.uint16)
+    vn = rng.integers(0, 65535, (R, L, B, W, H, D), dtype=np.uint16)
+    cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+    plg, flag = dev_i32(pl), torch.zeros(1, dtype=torch.int32, device="cuda")
+    das.das_kv_append(cache, dev_bf16(kn), dev_bf16(vn), dev_i32(acc), plg, flag)
+    torch.cuda.synchronize()
+    K2, V2, pl2, f2 = oracle.kv_append(K, V, kn, vn, acc, pl)
+    assert np.array_equal(host_bits(cache.k), K2) and np.array_equal(host_bits(cache.v), V2)
+    assert np.array_equal(plg.cpu().numpy(), pl2) and int(flag.item()) == f2
+    return f2
+
+
+def test_append_bit_exact_every_count():
+    """a = 0 (anchor only) .. a = W (all accepted), various offsets; every byte
+    of the cache, including sentinels around the written ranges, checked."""
+    W = 6
+    acc = np.array([0, 1, 3, W - 1, W, 2, 0], dtype=np.int32)
+    pl = np.array([0, 5, 17, 40, 0, 33, 49], dtype=np.int32)
+    assert _append_case(3, 2, 7, 50, 2, 64, W, pl, acc, 1) == 0
+
+
+def test_append_overflow_flags_and_skips():
+    acc = np.array([3, 0, 5], dtype=np.int32)
+    pl = np.array([30, 31, 20], dtype=np.int32)
+    assert _append_case(2, 1, 3, 32, 1, 128, 8, pl, acc, 2) == 1
+
+
+def test_verify_accept_append_chain_on_device():
+    """Verify -> accept -> append with no host round trip: accepted counts flow
+    from das_greedy_accept into das_kv_append on the device."""
+    import paper_2609_34538_gb300 as das
+    wl = wl_mod.WORKLOADS["verify"].replace(batch=3, layers=2, depths=4, key_depth=4,
+                                            value_depth=4, prefix=(90, 90), vocab=500)
+    W = wl.max_block
+    a_star, draft, logits = synth.accept_inputs(5, wl.batch, W, wl.vocab)
+    K, V = wl_mod.gen_cache(wl, depths=range(1, wl.depths + 1), tokens=90)
+    kn, vn = wl_mod.gen_staged(wl, W)
+    cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+    ws = das.new_workspace(cache, wl.q_heads, W)
+    pl = dev_i32(wl.prefix_lens())
+    bl = dev_i32(wl.block_lens())
+    q = dev_bf16(wl_mod.gen_q(wl, 1))
+    kb, vb = map(dev_bf16, wl_mod.gen_block_kv(wl, 1))
+    das.das_verify_attention(cache, 1, wl.depths, pl, bl, q, kb, vb, ws)
+    acc, tid, nxt = das.das_greedy_accept(torch.from_numpy(logits).cuda(),
+                                          torch.from_numpy(draft).cuda())
+    flag = torch.zeros(1, dtype=torch.int32, device="cuda")
+    das.das_kv_append(cache, dev_bf16(kn), dev_bf16(vn), acc, pl, flag)
+    torch.cuda.synchronize()
+    oa, _, _ = oracle.greedy_accept(logits, draft)
+    K2, V2, pl2, f2 = oracle.kv_append(K, V, kn, vn, oa, wl.prefix_lens())
+    assert np.array_equal(acc.cpu().numpy(), a_star)
+    assert np.array_equal(host_bits(cache.k), K2) and np.array_equal(host_bits(cache.v), V2)
+    assert np.array_equal(pl.cpu().numpy(), pl2) and int(flag.item()) == f2 == 0
