@@ -48,6 +48,9 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the workload's layer count (smaller profiling captures)")
+    ap.add_argument("--compact-depths", action="store_true",
+                    help="store 2 depths (key depth 1, value depth 2) instead of R: the same "
+                         "bytes per call in a smaller cache, for profiling captures")
     return ap.parse_args()
 
 
@@ -151,6 +154,8 @@ def gpu_arm(args):
     wl = wlm.WORKLOADS[args.workload]
     if args.layers:
         wl = wl.replace(layers=args.layers)
+    if args.compact_depths:
+        wl = wl.replace(depths=2, key_depth=1, value_depth=2)
     if wl.kind != "draft":
         raise SystemExit("the benchmark step needs a draft workload (its verify pass is derived)")
     R, L, B = wl.depths, wl.layers, wl.batch

@@ -71,8 +71,8 @@ typedef struct {
  * on the current device.  Returns 0 for shapes the kernels do not support.
  * The first 256 bytes of a workspace are a header; its first int32 is a
  * status word that the kernels OR with 1 if an internal wait ran out (a bug
- * guard; it stays set until the caller clears it).  Zero a new workspace
- * once before its first use.
+ * guard; it stays set until the caller clears it).  Zero a new workspace once
+ * before its first use.
  */
 size_t das_workspace_size(const das_kv_cache *cache, int num_q_heads, int max_block);
 

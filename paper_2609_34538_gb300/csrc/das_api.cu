@@ -99,8 +99,6 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
     p.q = static_cast<const uint16_t *>(q);
     p.out = static_cast<uint16_t *>(out);
     p.lse = lse;
-    uint8_t *ws = static_cast<uint8_t *>(workspace);
-    p.status = reinterpret_cast<int32_t *>(ws);
     p.B = c->batch;
     p.Hq = num_q_heads;
     p.Hkv = c->kv_heads;
@@ -113,12 +111,7 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
     const double scale = softmax_scale > 0.f ? (double)softmax_scale : 1.0 / sqrt((double)D);
     p.scale_log2 = (float)(scale * 1.4426950408889634);
     p.num_ctas = attn_grid_size(dev);
-    const size_t slots = (size_t)c->batch * c->kv_heads + (size_t)p.num_ctas;
-    size_t off = kWorkspaceHeader;
-    p.part_o = reinterpret_cast<float *>(ws + off);
-    off += slots * p.rows_max * D * sizeof(float);
-    off = (off + 255) & ~size_t(255);
-    p.part_lse = reinterpret_cast<float *>(ws + off);
+    attn_workspace_layout(workspace, c->batch, c->kv_heads, p.rows_max, D, p.num_ctas, p);
     return attn_launch(p, D, tk, tv, tkb, tvb, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? DAS_OK
                : DAS_ERR_CUDA;

@@ -32,7 +32,7 @@ struct AttnParams {
     float *lse;         // [B][Hq][max_block]
     float *part_o;      // [slots][rows_max][D]
     float *part_lse;    // [slots][rows_max]
-    int32_t *status;
+    int32_t *status;    // workspace status word
     int B, Hq, Hkv, G, max_block, rows_max, capacity;
     int key_slab, value_slab;  // (depth - 1) * layers + layer
     float scale_log2;          // softmax scale * log2(e)
@@ -42,8 +42,13 @@ struct AttnParams {
 // Number of CTAs the attention kernel launches on `device` (a persistent grid).
 int attn_grid_size(int device);
 size_t attn_workspace_bytes(int device, int batch, int kv_heads, int rows_max, int head_dim);
+// Carve a workspace into status word and partials (sets p.status, p.part_o,
+// p.part_lse).
+void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_max, int head_dim,
+                           int num_ctas, AttnParams &p);
 
-// Launch the split-K attention kernel and its merge on `stream`.
+// Launch the split-K attention kernel and its merge (a programmatic
+// dependent launch) on `stream`.
 cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
                         const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
                         const CUtensorMap &tm_vb, cudaStream_t stream);
