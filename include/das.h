@@ -177,6 +177,40 @@ das_status das_kv_append(const das_kv_cache *cache, const void *k_new, const voi
                          const int32_t *accepted, int W, int32_t *prefix_len,
                          int32_t *error_flag, void *stream);
 
+/*
+ * Bytes of device scratch built into the library for
+ * das_mature_v_attention_noalloc (32 MiB on every device that loads it).
+ */
+#define DAS_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+/*
+ * das_mature_v_attention without a caller-provided workspace.  The paper has
+ * no counterpart: this is for callers that cannot allocate device memory when
+ * they call (a fixed memory plan in a serving loop, a plugin that only
+ * receives the tensors it works on, a host that forbids cudaMalloc after
+ * start-up).  The split-K scratch is a fixed array of
+ * DAS_NOALLOC_SCRATCH_BYTES inside the library's device image, present on
+ * every device that loads the library until the process exits; this call
+ * allocates nothing and calls no allocating routine.
+ *   - Arguments and results as das_mature_v_attention, minus the workspace.
+ *   - Returns DAS_ERR_WORKSPACE if the shape needs more scratch than
+ *     DAS_NOALLOC_SCRATCH_BYTES (das_workspace_size() tells how much), with
+ *     nothing launched.
+ *   - The first call on a device looks up the array's device address (set-up
+ *     done once per device); make that first call before any CUDA graph
+ *     capture on that device.
+ *   - All calls share the array and it keeps the last call's contents: calls
+ *     that overlap in time on the GPU race and must be ordered by the caller.
+ *     Each call clears the status word at the array's head; the bits of a
+ *     call's device-side checks can be read there until the next call.
+ */
+das_status das_mature_v_attention_noalloc(const das_kv_cache *cache, int layer, int key_depth,
+                                          int value_depth, const int32_t *prefix_len,
+                                          const int32_t *block_len, int max_block, const void *q,
+                                          const void *k_blk, const void *v_blk, int num_q_heads,
+                                          float softmax_scale, void *out, float *lse,
+                                          void *stream);
+
 /* Static text for a status code. */
 const char *das_status_string(das_status s);
 

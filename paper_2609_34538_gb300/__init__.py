@@ -54,6 +54,8 @@ def _load():
     lib.das_greedy_accept.restype = i
     lib.das_kv_append.argtypes = [cp, p, p, p, i, p, p, p]
     lib.das_kv_append.restype = i
+    lib.das_mature_v_attention_noalloc.argtypes = [cp, i, i, i, p, p, i, p, p, p, i, f, p, p, p]
+    lib.das_mature_v_attention_noalloc.restype = i
     lib.das_status_string.argtypes = [i]
     lib.das_status_string.restype = ctypes.c_char_p
     return lib
@@ -168,6 +170,32 @@ def das_mature_v_attention(cache, layer, key_depth, value_depth, prefix_len, blo
         _ptr(block_len), T, _ptr(q), _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale),
         _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(stream)),
         "das_mature_v_attention")
+    return out, lse
+
+
+def das_mature_v_attention_noalloc(cache, layer, key_depth, value_depth, prefix_len, block_len, q,
+                                   k_blk, v_blk, out=None, lse=None, softmax_scale=0.0,
+                                   stream=None):
+    """das_mature_v_attention for callers that cannot allocate device memory:
+    the split-K scratch is a fixed array inside the library (shared by every
+    call on a device; calls that overlap on the GPU race).  `out` and `lse`
+    must be given by such callers; they are allocated here only for
+    convenience when omitted."""
+    R, L, B, cap, H, D = cache.shape
+    T, Hq = q.shape[1], q.shape[2]
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((B, Hq, T), dtype=torch.float32, device=q.device)
+    _need(prefix_len, torch.int32, "prefix_len", 1)
+    _need(block_len, torch.int32, "block_len", 1)
+    for t, n in ((q, "q"), (k_blk, "k_blk"), (v_blk, "v_blk"), (out, "out")):
+        _need(t, torch.bfloat16, n, 4)
+    _need(lse, torch.float32, "lse", 3)
+    _check(LIB.das_mature_v_attention_noalloc(
+        ctypes.byref(cache.desc), layer, key_depth, value_depth, _ptr(prefix_len),
+        _ptr(block_len), T, _ptr(q), _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale),
+        _ptr(out), _ptr(lse), _stream(stream)), "das_mature_v_attention_noalloc")
     return out, lse
 
 
