@@ -29,9 +29,10 @@ EncodeTiledFn encode_fn() {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// bf16 tensor map over `rank` dims (innermost first) with a {64, 1, 64, 1..}
-// box and 128-byte swizzle: one box is 64 positions x 64 head_dim elements.
-bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims) {
+// bf16 tensor map over `rank` dims (innermost first) with 128-byte swizzle;
+// the default box {64, 1, 64, 1, 1} is 64 positions x 64 head_dim elements.
+bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
+                 const cuuint32_t *box_in = nullptr) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t strides[4];
@@ -41,6 +42,8 @@ bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims) {
         strides[i] = s;
     }
     cuuint32_t box[5] = {64, 1, 64, 1, 1};
+    if (box_in)
+        for (int i = 0; i < rank; ++i) box[i] = box_in[i];
     cuuint32_t estr[5] = {1, 1, 1, 1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, base, dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -93,6 +96,17 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
         !encode_bf16(&tvb, const_cast<void *>(v_blk), 4, blk_dims))
         return DAS_ERR_CUDA;
 
+    // queries: rows of one pair are heads h*G .. h*G+G-1 of every block row i,
+    // i.e. a {64, G, max_block, 1} box over [B][max_block][Hq][D]
+    const bool use_tc = true;
+    CUtensorMap tq;
+    if (use_tc) {
+        const cuuint64_t q_dims[4] = {(cuuint64_t)D, (cuuint64_t)num_q_heads,
+                                      (cuuint64_t)max_block, (cuuint64_t)c->batch};
+        const cuuint32_t q_box[4] = {64, (cuuint32_t)G, (cuuint32_t)max_block, 1};
+        if (!encode_bf16(&tq, const_cast<void *>(q), 4, q_dims, q_box)) return DAS_ERR_CUDA;
+    }
+
     AttnParams p;
     p.prefix_len = prefix_len;
     p.block_len = block_len;
@@ -110,11 +124,12 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
     p.value_slab = (value_depth - 1) * c->layers + layer;
     const double scale = softmax_scale > 0.f ? (double)softmax_scale : 1.0 / sqrt((double)D);
     p.scale_log2 = (float)(scale * 1.4426950408889634);
-    p.num_ctas = attn_grid_size(dev);
+    p.num_ctas = use_tc ? attn_tc_grid_size(dev) : attn_grid_size(dev);
     attn_workspace_layout(workspace, c->batch, c->kv_heads, p.rows_max, D, p.num_ctas, p);
-    return attn_launch(p, D, tk, tv, tkb, tvb, static_cast<cudaStream_t>(stream)) == cudaSuccess
-               ? DAS_OK
-               : DAS_ERR_CUDA;
+    const cudaError_t e =
+        use_tc ? attn_tc_launch(p, D, tk, tv, tkb, tvb, tq, static_cast<cudaStream_t>(stream))
+               : attn_launch(p, D, tk, tv, tkb, tvb, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? DAS_OK : DAS_ERR_CUDA;
 }
 
 }  // namespace

@@ -863,6 +863,9 @@ template <int D>
 constexpr int kStages = (D == 128) ? 3 : 6;
 
 template <int D>
+cudaError_t merge_launch_d(const AttnParams &p, cudaStream_t stream);
+
+template <int D>
 cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
                      const CUtensorMap &tkb, const CUtensorMap &tvb, cudaStream_t stream) {
     constexpr int ST = kStages<D>;
@@ -880,6 +883,11 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
     attn_kernel<D, ST><<<p.num_ctas, kThreads, smem, stream>>>(tk, tv, tkb, tvb, p);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    return merge_launch_d<D>(p, stream);
+}
+
+template <int D>
+cudaError_t merge_launch_d(const AttnParams &p, cudaStream_t stream) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(p.B * p.Hkv * ((p.rows_max + kConsumerWarps - 1) / kConsumerWarps)));
     cfg.blockDim = dim3(kThreads);
@@ -923,6 +931,12 @@ void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_ma
     off += slots * rows_max * head_dim * sizeof(float);
     off = (off + 255) & ~size_t(255);
     p.part_lse = reinterpret_cast<float *>(ws + off);
+}
+
+cudaError_t attn_merge_launch(const AttnParams &p, int head_dim, cudaStream_t stream) {
+    if (head_dim == 128) return merge_launch_d<128>(p, stream);
+    if (head_dim == 64) return merge_launch_d<64>(p, stream);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,

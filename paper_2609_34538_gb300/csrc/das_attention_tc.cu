@@ -1,0 +1,784 @@
+// das_attention_tc.cu -- depth-asynchronous attention (Eqs. 2-3, Sec. 3.2) and
+// the full-depth verify attention (Sec. 3.4) on the 5th-generation tensor
+// cores of sm_103a (tcgen05, accumulators in tensor memory).
+//
+// Work decomposition is that of das_attention.cu: every (sequence, kv head)
+// pair owns ceil(P/64) prefix tiles plus one block tile, all pairs' tiles form
+// one list, CTA c of a persistent grid (one CTA per SM) takes the range
+// [c N / C, (c+1) N / C), cut into segments at pair boundaries; a segment that
+// covers its pair writes the output, the others write partials that
+// merge_kernel combines.
+//
+// One CTA = one control warp + four softmax warps.
+//   control (warp 4, one lane): TMA loads of 64-key K and V tiles STAGES ahead
+//     into a ring of shared-memory stages, TMA loads of each segment's query
+//     rows (the pair's G * max_block rows, rows ordered i * G + g, which is the
+//     order of a {64, G, max_block} box), and the MMAs:
+//       S = Q K^T    tcgen05.mma M=64 N=64 K=D   -> S buffer (k % 2) in TMEM
+//       O += P V     tcgen05.mma M=64 N=D K=64   -> O in TMEM
+//     S of tile k+1 is issued before P V of tile k, so the tensor core works on
+//     the next tile while the softmax warps handle the current one.  A stage is
+//     refilled once the P V that read it has completed.
+//   softmax warps: warp w owns rows 16w..16w+15, which an M=64 MMA places in
+//     TMEM lanes 32w..32w+15.  Each thread loads its row's 64 scores, masks and
+//     scales them (base 2), keeps a reference max m that only moves when a
+//     score exceeds it by more than 8 (then O and l are rescaled in TMEM),
+//     writes P = 2^(s - m) as bf16 into a 128-byte-swizzled [64 rows][64 keys]
+//     buffer (the K-major A operand of P V) and accumulates l.  At the end of a
+//     segment it reads its O row from TMEM and writes O / l and the lse.
+// Every wait is bounded (2 s); a time-out sets the status word and stops the
+// CTA's waits.  Tensor memory (256 columns) is freed before the CTA exits.
+#include <cuda_bf16.h>
+
+#include "das_internal.h"
+
+namespace das {
+namespace tc {
+namespace {
+
+constexpr uint32_t kFull = 0xffffffffu;
+constexpr unsigned long long kWaitNs = 2000000000ull;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kStages = 4;
+constexpr int kSoftWarps = 4;
+constexpr int kProducerWarp = kSoftWarps;     // TMA loads
+constexpr int kMmaWarp = kSoftWarps + 1;      // tcgen05 MMAs
+constexpr int kThreads = (kSoftWarps + 2) * 32;
+constexpr int kRows = 64;            // M of every MMA (query rows per pair)
+constexpr int kTmemCols = 256;       // S buffers [0, 128), O [128, 128 + D)
+constexpr float kRescaleLog2 = 8.f;  // move the reference max only beyond 2^8
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ unsigned long long globaltimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait; false after 2 s or once another thread of the CTA gave up.
+__device__ __noinline__ bool wait_slow(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                       int32_t *status) {
+    const unsigned long long t0 = globaltimer();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((it & 63u) == 0) {
+            if (*abort_flag) return false;
+            if (globaltimer() - t0 > kWaitNs) {
+                *abort_flag = 1;
+                atomicOr(status, kStatusWaitTimeout);
+                return false;
+            }
+        }
+    }
+}
+__device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                     int32_t *status) {
+#pragma unroll 1
+    for (int i = 0; i < 8; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    return wait_slow(bar, parity, abort_flag, status);
+}
+
+__device__ __forceinline__ void tma_5d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
+                                       int c1, int c2, int c3, int c4, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        ".L2::cache_hint [%0], [%1, {%3, %4, %5, %6, %7}], [%2], %8;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
+        "r"(c4), "l"(policy)
+        : "memory");
+}
+__device__ __forceinline__ void tma_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
+                                       int c1, int c2, int c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+        : "memory");
+}
+
+// ---- tcgen05 ----------------------------------------------------------------
+// Shared-memory matrix descriptor: start, leading / stride byte offsets,
+// descriptor version 1, layout 2 = 128-byte swizzle.
+__device__ __forceinline__ uint64_t sdesc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((addr >> 4) & 0x3FFF) | (uint64_t)((lbo >> 4) & 0x3FFF) << 16 |
+           (uint64_t)((sbo >> 4) & 0x3FFF) << 32 | (uint64_t)1 << 46 | (uint64_t)2 << 61;
+}
+// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, majors, N, M.
+__host__ __device__ constexpr uint32_t idesc(int M, int N, int a_mn_major, int b_mn_major) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn_major << 15) |
+           ((uint32_t)b_mn_major << 16) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id,
+                                    uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(id), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// true on exactly one lane of the (converged) warp
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred;
+    asm volatile(
+        "{\n .reg .pred P;\n .reg .b32 R;\n elect.sync R|P, 0xffffffff;\n"
+        " selp.u32 %0, 1, 0, P;\n}\n"
+        : "=r"(pred));
+    return pred != 0;
+}
+// 32 lanes x 32 consecutive 32-bit columns; thread t gets lane (base + t).
+// The load and its wait form one statement, so no use of the registers can
+// be scheduled before the data is there.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%16];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+            taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+        "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+        "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+        "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+        "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+        "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+        "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+        "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+// ---- tile list (as in das_attention.cu) ---------------------------------------
+__device__ __forceinline__ int clamp_prefix(const AttnParams &p, int b) {
+    int v = p.prefix_len[b];
+    return v < 0 ? 0 : (v > p.capacity ? p.capacity : v);
+}
+__device__ __forceinline__ int clamp_block(const AttnParams &p, int b) {
+    int v = p.block_len[b];
+    return v < 0 ? 0 : (v > p.max_block ? p.max_block : v);
+}
+__device__ __forceinline__ int tiles_of(int P) { return (P + kTileKeys - 1) / kTileKeys + 1; }
+__device__ __forceinline__ long long range_lo(int c, long long N, int C) {
+    return (long long)c * N / C;
+}
+
+struct Walk {
+    int b, h, t, nt, P, T;
+};
+__device__ __forceinline__ void walk_load_seq(const AttnParams &p, Walk &w) {
+    if (w.b < p.B) {
+        w.P = clamp_prefix(p, w.b);
+        w.T = clamp_block(p, w.b);
+        w.nt = tiles_of(w.P);
+    }
+}
+__device__ __forceinline__ void walk_next(const AttnParams &p, Walk &w) {
+    if (++w.t == w.nt) {
+        w.t = 0;
+        if (++w.h == p.Hkv) {
+            w.h = 0;
+            ++w.b;
+            walk_load_seq(p, w);
+        }
+    }
+}
+
+// Range of this CTA and its first position (a whole warp executes this).
+__device__ bool plan(const AttnParams &p, long long &N, long long &lo, long long &hi, Walk &w) {
+    const int lane = threadIdx.x & 31;
+    long long before = 0, total = 0;
+    // pass 1: N
+    for (int b0 = 0; b0 < p.B; b0 += 32) {
+        const int b = b0 + lane;
+        total += b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
+    }
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) total += __shfl_xor_sync(kFull, total, d);
+    N = total;
+    lo = range_lo(blockIdx.x, N, p.num_ctas);
+    hi = range_lo(blockIdx.x + 1, N, p.num_ctas);
+    if (lo >= hi) return false;
+    // pass 2: the sequence holding lo
+    long long run = 0;
+    w.b = p.B;
+    for (int b0 = 0; b0 < p.B; b0 += 32) {
+        const int b = b0 + lane;
+        const long long v = b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
+        long long inc = v;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const long long t = __shfl_up_sync(kFull, inc, d);
+            if (lane >= d) inc += t;
+        }
+        const long long tot = __shfl_sync(kFull, inc, 31);
+        if (run + tot > lo) {
+            const int first = __ffs(__ballot_sync(kFull, run + inc > lo)) - 1;
+            before = run + __shfl_sync(kFull, inc - v, first);
+            w.b = b0 + first;
+            break;
+        }
+        run += tot;
+    }
+    walk_load_seq(p, w);
+    const long long off = lo - before;
+    w.h = (int)(off / w.nt);
+    w.t = (int)(off % w.nt);
+    return true;
+}
+
+template <int D>
+struct Layout {
+    static constexpr int kPanels = D / 64;
+    static constexpr int kTileBytes = kTileKeys * D * 2;  // K or V of one tile
+    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kQBytes = kPanels * kRows * 128;  // one query buffer
+    static constexpr int kPBytes = kRows * kTileKeys * 2;  // one P buffer
+    static constexpr int kStagesOff = 0;
+    static constexpr int kQOff = kStages * kStageBytes;
+    static constexpr int kPOff = kQOff + 2 * kQBytes;
+    static constexpr int kBarOff = kPOff + 2 * kPBytes;
+    // barriers: full[kStages], empty[kStages], qfull[2], qempty[2], sready[2],
+    // sfree[2], pready[2], pvdone, drain
+    static constexpr int kNumBars = 2 * kStages + 12;
+    static constexpr int kMiscOff = kBarOff + kNumBars * 8;
+    static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
+};
+
+// K-major 128B-swizzled address of bf16 element (row, col) of a [64][64] panel
+__device__ __forceinline__ uint32_t p_chunk_addr(uint32_t base, int row, int chunk) {
+    return base + row * 128 + ((chunk ^ (row & 7)) << 4);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ CUtensorMap tm_kb,
+                   const __grid_constant__ CUtensorMap tm_vb,
+                   const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
+    using Lt = Layout<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~uintptr_t(1023));
+    const uint32_t sbase = smem_u32(sm);
+    const uint32_t bars = sbase + Lt::kBarOff;
+    const uint32_t b_full = bars, b_empty = bars + 8 * kStages, b_qfull = b_empty + 8 * kStages,
+                   b_qempty = b_qfull + 16, b_sready = b_qempty + 16, b_sfree = b_sready + 16,
+                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 8;
+    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(sm + Lt::kMiscOff);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Lt::kMiscOff + 4);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (blockIdx.x == 0 && threadIdx.x == 0)
+        for (int b = 0; b < p.B; ++b)
+            if (p.prefix_len[b] != clamp_prefix(p, b) || p.block_len[b] != clamp_block(p, b))
+                atomicOr(p.status, kStatusClamped);
+    long long N, lo, hi;
+    Walk w0;
+    if (!plan(p, N, lo, hi, w0)) return;  // uniform across the CTA
+    const long long ntiles = hi - lo;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(b_full + 8 * s, 1);
+            mbar_init(b_empty + 8 * s, 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(b_qfull + 8 * i, 1);
+            mbar_init(b_qempty + 8 * i, 1);
+            mbar_init(b_sready + 8 * i, 1);
+            mbar_init(b_sfree + 8 * i, kSoftWarps);
+            mbar_init(b_pready + 8 * i, kSoftWarps);
+        }
+        mbar_init(b_pvdone, 1);
+        mbar_init(b_drain, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile(
+            "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                smem_u32(const_cast<uint32_t *>(tmem_slot))),
+            "n"(kTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    fence_before();
+    __syncthreads();
+    fence_after();
+    const uint32_t tmem = *tmem_slot;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    if (warp == kProducerWarp) {
+        // ================================ producer ===============================
+        // Warp-uniform loop; one elected lane issues.  Stage s is reused once
+        // the P V that read it has completed (the MMA warp commits empty[s]);
+        // a query buffer once the last S of the segment before last completed.
+        uint64_t policy;
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+        if (elect_one()) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k))
+                         : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v))
+                         : "memory");
+        }
+        Walk wl = w0;
+        int qseg = -1;
+        bool ok = true;
+        for (long long j = 0; j < ntiles && ok; ++j) {
+            if (j == 0 || wl.t == 0) {  // the segment's query rows
+                ++qseg;
+                const int qb = qseg & 1;
+                if (qseg >= 2)
+                    ok = ok && wait(b_qempty + 8 * qb, (uint32_t)(((qseg - 2) >> 1) & 1),
+                                    abort_flag, p.status);
+                if (ok && elect_one()) {
+                    const uint32_t full = b_qfull + 8 * qb;
+                    const uint32_t dst = sbase + Lt::kQOff + qb * Lt::kQBytes;
+                    mbar_arrive_expect_tx(full, Lt::kPanels * p.rows_max * 128);
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp)
+                        tma_4d(dst + dp * (kRows * 128), &tm_q, full, dp * 64, wl.h * p.G, 0,
+                               wl.b);
+                }
+            }
+            const int s = (int)(j % kStages);
+            if (j >= kStages)
+                ok = ok && wait(b_empty + 8 * s, (uint32_t)(((j - kStages) / kStages) & 1),
+                                abort_flag, p.status);
+            if (ok && elect_one()) {
+                const uint32_t full = b_full + 8 * s;
+                const uint32_t kdst = sbase + Lt::kStagesOff + s * Lt::kStageBytes;
+                const uint32_t vdst = kdst + Lt::kTileBytes;
+                mbar_arrive_expect_tx(full, Lt::kStageBytes);
+                if (wl.t < wl.nt - 1) {
+                    const int tok = wl.t * kTileKeys;
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                        tma_5d(kdst + dp * 8192, &tm_k, full, dp * 64, wl.h, tok, wl.b,
+                               p.key_slab, policy);
+                        tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
+                               p.value_slab, policy);
+                    }
+                } else {
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                        tma_4d(kdst + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
+                        tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
+                    }
+                }
+            }
+            __syncwarp();
+            walk_next(p, wl);
+        }
+    } else if (warp == kMmaWarp) {
+        // ================================== MMA ==================================
+        const uint32_t id_s = idesc(kRows, kTileKeys, 0, 0);
+        const uint32_t id_pv = idesc(kRows, D, 0, 1);
+        // descriptors are affine in the address: build each base once and add
+        // (byte offset >> 4) for buffers and k-steps
+        const uint64_t dq0 = sdesc(sbase + Lt::kQOff, 16, 1024);
+        const uint64_t dk0 = sdesc(sbase + Lt::kStagesOff, 16, 1024);
+        const uint64_t dv0 = sdesc(sbase + Lt::kStagesOff + Lt::kTileBytes, 8192, 1024);
+        const uint64_t dp0 = sdesc(sbase + Lt::kPOff, 16, 1024);
+        Walk wsn = w0;  // walk of the next S
+        int qseg = -1, qcur = 0;
+        bool ok = true;
+        auto next_s = [&](long long kn) {  // S of tile kn, two tiles ahead of P V
+            if (kn == 0 || wsn.t == 0) {
+                ++qseg;
+                qcur = qseg & 1;
+                ok = ok && wait(b_qfull + 8 * qcur, (uint32_t)((qseg >> 1) & 1), abort_flag,
+                                p.status);
+            }
+            const int s = (int)(kn % kStages);
+            ok = ok && wait(b_full + 8 * s, (uint32_t)((kn / kStages) & 1), abort_flag, p.status);
+            if (kn >= 2)
+                ok = ok && wait(b_sfree + 8 * (int)(kn & 1), (uint32_t)(((kn - 2) >> 1) & 1),
+                                abort_flag, p.status);
+            const bool seg_end = (wsn.t == wsn.nt - 1) || (kn + 1 == ntiles);
+            if (ok) {
+                fence_after();
+                if (elect_one()) {
+                    const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
+                    const uint64_t b0 = dk0 + (uint64_t)((s * Lt::kStageBytes) >> 4);
+                    const uint32_t dS = tmem + (uint32_t)((kn & 1) * kTileKeys);
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        // panel kk / 4, then 16 elements (32 bytes) within the 128-byte row
+                        const uint32_t qoff = ((kk >> 2) * (kRows * 128) + (kk & 3) * 32) >> 4;
+                        const uint32_t koff = ((kk >> 2) * 8192 + (kk & 3) * 32) >> 4;
+                        mma(dS, a0 + qoff, b0 + koff, id_s, kk > 0);
+                    }
+                    mma_commit(b_sready + 8 * (int)(kn & 1));
+                    if (seg_end) mma_commit(b_qempty + 8 * qcur);
+                }
+                __syncwarp();
+            }
+            walk_next(p, wsn);
+        };
+        for (long long kn = 0; kn < 2 && kn < ntiles && ok; ++kn) next_s(kn);
+        Walk wm = w0;  // tile of the next P V
+        for (long long k = 0; k < ntiles && ok; ++k) {
+            const bool first = (k == 0) || (wm.t == 0);
+            ok = ok && wait(b_pready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1), abort_flag,
+                            p.status);
+            if (!ok) break;
+            fence_after();
+            if (elect_one()) {
+                const int s = (int)(k % kStages);
+                const uint64_t a0 = dp0 + (uint64_t)(((k & 1) * Lt::kPBytes) >> 4);
+                const uint64_t b0 = dv0 + (uint64_t)((s * Lt::kStageBytes) >> 4);
+                const uint32_t dO = tmem + 2 * kTileKeys;
+#pragma unroll
+                for (int kk = 0; kk < kTileKeys / 16; ++kk)
+                    mma(dO, a0 + (uint64_t)((kk * 32) >> 4), b0 + (uint64_t)((kk * 2048) >> 4),
+                        id_pv, (!first || kk > 0) ? 1u : 0u);
+                mma_commit(b_pvdone);
+                mma_commit(b_empty + 8 * s);
+            }
+            __syncwarp();
+            if (k + 2 < ntiles) next_s(k + 2);
+            walk_next(p, wm);
+        }
+        // all MMAs issued here are complete before tensor memory is freed
+        // (only a timed-out run can leave any in flight)
+        if (elect_one()) mma_commit(b_drain);
+        __syncwarp();
+        const unsigned long long t0 = globaltimer();
+        while (!mbar_try_wait(b_drain, 0) && globaltimer() - t0 < kWaitNs) {
+        }
+    } else {
+        // ================================ softmax ================================
+        const int row = warp * 16 + lane;  // meaningful for lane < 16
+        const bool owner = lane < 16;
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        Walk ws = w0;
+        float m_ref = -INFINITY, l_sum = 0.f;
+        int rows_active = 0, irow = 0;
+        long long seg_first = lo;
+        for (long long k = 0; k < ntiles; ++k) {
+            const bool first = (k == 0) || (ws.t == 0);
+            const bool block_tile = ws.t == ws.nt - 1;
+            const bool last = block_tile || (k + 1 == ntiles);
+            if (first) {
+                m_ref = -INFINITY;
+                l_sum = 0.f;
+                rows_active = p.G * ws.T;
+                irow = row / p.G;
+                seg_first = lo + k;
+            }
+            const int nvalid = block_tile ? ws.T : min(kTileKeys, ws.P - ws.t * kTileKeys);
+            const int s = (int)(k % kStages);
+            // ---- scores: two compact passes over 16-column chunks of S ----
+            const bool ok_s = wait(b_sready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1),
+                                   abort_flag, p.status);
+            fence_after();
+            const uint32_t s_addr = tmem + lane_base + (uint32_t)((k & 1) * kTileKeys);
+            const bool valid_row = owner && row < rows_active && ok_s;
+            // keys j < lim are visible to this row; a full prefix tile needs no
+            // mask (rows of other lanes are computed but never stored)
+            const int lim = !valid_row ? 0 : (block_tile ? min(nvalid, irow + 1) : nvalid);
+            const bool full_tile = !block_tile && nvalid == kTileKeys;
+            const float scale = p.scale_log2;
+            // first tile of a segment: the reference max comes from a max pass
+            if (first) {
+                float mt = -INFINITY;
+#pragma unroll 1
+                for (int c = 0; c < kTileKeys; c += 16) {
+                    float v[16];
+                    tmem_ld16(s_addr + c, v);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        mt = fmaxf(mt, c + j < lim ? v[j] * scale : -INFINITY);
+                }
+                m_ref = mt;
+            }
+            // O and the P buffer of tile k-2 are free once P V of tile k-1 is done
+            if (k >= 1) wait(b_pvdone, (uint32_t)((k - 1) & 1), abort_flag, p.status);
+            fence_after();
+            // P = 2^(s - m) as bf16 into the swizzled P buffer (16 keys = 2 chunks),
+            // with the tile max on the side; a second pass only if the max moved
+            // beyond the reference by more than 2^8
+            const uint32_t pbuf = sbase + Lt::kPOff + (uint32_t)((k & 1) * Lt::kPBytes);
+            float lt = 0.f;
+#pragma unroll 1
+            for (int pass = 0; pass < 2; ++pass) {
+                const float mu = m_ref == -INFINITY ? 0.f : m_ref;
+                float mt = -INFINITY;
+                lt = 0.f;
+#pragma unroll 1
+                for (int c = 0; c < kTileKeys; c += 16) {
+                    float v[16];
+                    tmem_ld16(s_addr + c, v);
+                    uint32_t w[8];
+                    if (full_tile) {  // warp-uniform: no masks
+                        float vm = v[0];
+#pragma unroll
+                        for (int j = 1; j < 16; ++j) vm = fmaxf(vm, v[j]);
+                        mt = fmaxf(mt, vm * scale);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const float a = ex2(fmaf(v[2 * e], scale, -mu));
+                            const float b2 = ex2(fmaf(v[2 * e + 1], scale, -mu));
+                            lt += a + b2;
+                            w[e] = pack_bf16(a, b2);
+                        }
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const float x0 = c + 2 * e < lim ? v[2 * e] * scale : -INFINITY;
+                            const float x1 = c + 2 * e + 1 < lim ? v[2 * e + 1] * scale : -INFINITY;
+                            mt = fmaxf(mt, fmaxf(x0, x1));
+                            const float a = ex2(x0 - mu), b2 = ex2(x1 - mu);
+                            lt += a + b2;
+                            w[e] = pack_bf16(a, b2);
+                        }
+                    }
+                    if (owner) {
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                         p_chunk_addr(pbuf, row, c / 8)),
+                                     "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                     : "memory");
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                         p_chunk_addr(pbuf, row, c / 8 + 1)),
+                                     "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                                     : "memory");
+                    }
+                }
+                const bool jump = valid_row && !first && mt > m_ref + kRescaleLog2;
+                if (!__any_sync(kFull, jump)) break;
+                // the max moved: rescale O and l to the new reference, redo P
+                const float alpha = jump ? ex2(m_ref - mt) : 1.f;  // m_ref -inf gives 0
+                if (jump) {
+                    m_ref = mt;
+                    l_sum *= alpha;
+                }
+#pragma unroll 1
+                for (int c = 0; c < D; c += 32) {
+                    float v[32];
+                    const uint32_t ta = tmem + lane_base + (uint32_t)(2 * kTileKeys + c);
+                    tmem_ld32(ta, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] *= alpha;
+                    tmem_st32(ta, v);
+                }
+            }
+            // S of this tile is no longer read: its buffer may take tile k+2
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_sfree + 8 * (int)(k & 1));
+            l_sum += lt;
+            // keys past the end of the tile may hold anything: zero their V rows
+            if (nvalid < kTileKeys) {
+                const uint32_t vt = sbase + Lt::kStagesOff + s * Lt::kStageBytes + Lt::kTileBytes;
+                const int nzero = (kTileKeys - nvalid) * 8 * Lt::kPanels;  // 16-byte chunks
+                for (int i = threadIdx.x; i < nzero; i += kSoftWarps * 32) {
+                    const int panel = i / ((kTileKeys - nvalid) * 8);
+                    const int rem = i % ((kTileKeys - nvalid) * 8);
+                    const int key = nvalid + rem / 8, chunk = rem % 8;
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                     vt + panel * 8192 + key * 128 + (chunk << 4)),
+                                 "r"(0u)
+                                 : "memory");
+                }
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
+
+            // ---- end of segment: O / l and lse ----
+            if (last) {
+                wait(b_pvdone, (uint32_t)(k & 1), abort_flag, p.status);
+                fence_after();
+                const long long pair_first = lo + k - ws.t;
+                const bool whole = (seg_first == pair_first) && block_tile;
+                const int pair = ws.b * p.Hkv + ws.h;
+                const size_t slot = (size_t)pair + blockIdx.x;
+                const bool write = owner && row < rows_active;
+                const float inv = l_sum > 0.f ? 1.f / l_sum : 0.f;
+                const float lse =
+                    l_sum > 0.f ? (m_ref + __log2f(l_sum)) * kLn2 : -INFINITY;
+                const int gq = row % p.G;
+                uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
+                                          (size_t)ws.h * p.G + gq) * D;
+                float *prow = p.part_o + (slot * p.rows_max + row) * D;
+#pragma unroll 1
+                for (int c = 0; c < D; c += 32) {
+                    float v[32];
+                    tmem_ld32(tmem + lane_base + (uint32_t)(2 * kTileKeys + c), v);
+                    if (write) {
+                        if (whole) {
+#pragma unroll
+                            for (int j = 0; j < 32; j += 8)
+                                *reinterpret_cast<uint4 *>(orow + c + j) =
+                                    make_uint4(pack_bf16(v[j] * inv, v[j + 1] * inv),
+                                               pack_bf16(v[j + 2] * inv, v[j + 3] * inv),
+                                               pack_bf16(v[j + 4] * inv, v[j + 5] * inv),
+                                               pack_bf16(v[j + 6] * inv, v[j + 7] * inv));
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; j += 4)
+                                *reinterpret_cast<float4 *>(prow + c + j) =
+                                    make_float4(v[j] * inv, v[j + 1] * inv, v[j + 2] * inv,
+                                                v[j + 3] * inv);
+                        }
+                    }
+                }
+                if (write) {
+                    if (whole)
+                        p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gq) * p.max_block +
+                              irow] = lse;
+                    else
+                        p.part_lse[slot * p.rows_max + row] = lse;
+                }
+                if (whole) {  // rows past the block: 0 and lse -inf
+                    for (int idx = threadIdx.x; idx < (p.rows_max - rows_active) * (D / 8);
+                         idx += kSoftWarps * 32) {
+                        const int r = rows_active + idx / (D / 8), col = (idx % (D / 8)) * 8;
+                        const int ii = r / p.G, gg = r % p.G;
+                        *reinterpret_cast<uint4 *>(p.out + (((size_t)ws.b * p.max_block + ii) *
+                                                                 p.Hq +
+                                                             (size_t)ws.h * p.G + gg) * D + col) =
+                            make_uint4(0u, 0u, 0u, 0u);
+                        if (col == 0)
+                            p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gg) * p.max_block +
+                                  ii] = -INFINITY;
+                    }
+                }
+                fence_before();
+            }
+            walk_next(p, ws);
+        }
+    }
+    // every MMA was waited on by the control lane and the softmax warps
+    fence_before();
+    __syncthreads();
+    fence_after();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "n"(kTmemCols));
+}
+
+}  // namespace
+
+template <int D>
+cudaError_t launch_tc_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
+                        const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
+                        cudaStream_t stream) {
+    constexpr int smem = Layout<D>::kBytes;
+    static bool configured[64] = {false};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 64 && !configured[dev]) {
+        e = cudaFuncSetAttribute(attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 smem);
+        if (e != cudaSuccess) return e;
+        configured[dev] = true;
+    }
+    attn_tc_kernel<D><<<p.num_ctas, kThreads, smem, stream>>>(tk, tv, tkb, tvb, tq, p);
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+
+int attn_tc_grid_size(int device) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
+        return 0;
+    return sms;
+}
+
+cudaError_t attn_tc_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
+                           const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
+                           const CUtensorMap &tm_vb, const CUtensorMap &tm_q,
+                           cudaStream_t stream) {
+    cudaError_t e;
+    if (head_dim == 128)
+        e = tc::launch_tc_d<128>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+    else if (head_dim == 64)
+        e = tc::launch_tc_d<64>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+    else
+        return cudaErrorInvalidValue;
+    if (e != cudaSuccess) return e;
+    return attn_merge_launch(p, head_dim, stream);
+}
+
+}  // namespace das

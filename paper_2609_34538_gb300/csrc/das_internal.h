@@ -53,6 +53,17 @@ cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm
                         const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
                         const CUtensorMap &tm_vb, cudaStream_t stream);
 
+// The merge of split pairs alone (a programmatic dependent launch).
+cudaError_t attn_merge_launch(const AttnParams &p, int head_dim, cudaStream_t stream);
+
+// The tcgen05 attention kernel (one CTA per SM) and its merge on `stream`;
+// tm_q maps the queries [B][max_block][Hq][D] with a {64, G, max_block, 1} box.
+int attn_tc_grid_size(int device);
+cudaError_t attn_tc_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
+                           const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
+                           const CUtensorMap &tm_vb, const CUtensorMap &tm_q,
+                           cudaStream_t stream);
+
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream);
