@@ -179,6 +179,23 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
+// 16 lanes x 2 halves: thread t < 16 gets lane t, columns [c, c + 16); thread
+// t + 16 gets lane t, columns [c + 32, c + 48).  With M = 64 a warp's rows sit
+// in its first 16 lanes, so two threads share each row.
+__device__ __forceinline__ void tmem_ld_half16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15}, [%16], 32;\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
     uint32_t r[16];
     asm volatile(
@@ -314,8 +331,8 @@ struct Layout {
     static constexpr int kPOff = kQOff + 2 * kQBytes;
     static constexpr int kBarOff = kPOff + 2 * kPBytes;
     // barriers: full[kStages], empty[kStages], qfull[2], qempty[2], sready[2],
-    // sfree[2], pready[2], pvdone, drain
-    static constexpr int kNumBars = 2 * kStages + 12;
+    // sfree[2], pready[2], pvdone[2], drain
+    static constexpr int kNumBars = 2 * kStages + 13;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
 };
@@ -340,7 +357,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t bars = sbase + Lt::kBarOff;
     const uint32_t b_full = bars, b_empty = bars + 8 * kStages, b_qfull = b_empty + 8 * kStages,
                    b_qempty = b_qfull + 16, b_sready = b_qempty + 16, b_sfree = b_sready + 16,
-                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 8;
+                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 16;
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(sm + Lt::kMiscOff);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Lt::kMiscOff + 4);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -367,6 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(b_pready + 8 * i, kSoftWarps);
         }
         mbar_init(b_pvdone, 1);
+        mbar_init(b_pvdone + 8, 1);
         mbar_init(b_drain, 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -509,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int kk = 0; kk < kTileKeys / 16; ++kk)
                     mma(dO, a0 + (uint64_t)((kk * 32) >> 4), b0 + (uint64_t)((kk * 2048) >> 4),
                         id_pv, (!first || kk > 0) ? 1u : 0u);
-                mma_commit(b_pvdone);
+                mma_commit(b_pvdone + 8 * (int)(k & 1));
                 mma_commit(b_empty + 8 * s);
             }
             __syncwarp();
@@ -525,7 +543,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // ================================ softmax ================================
-        const int row = warp * 16 + lane;  // meaningful for lane < 16
+        // thread (warp, lane) handles row 16 warp + lane % 16, keys of its half
+        // (lane / 16) of each tile; the epilogue's O rows are read by lanes < 16
+        const int row = warp * 16 + (lane & 15);
+        const int half = lane >> 4;
         const bool owner = lane < 16;
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         Walk ws = w0;
@@ -550,7 +571,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                    abort_flag, p.status);
             fence_after();
             const uint32_t s_addr = tmem + lane_base + (uint32_t)((k & 1) * kTileKeys);
-            const bool valid_row = owner && row < rows_active && ok_s;
+            const bool valid_row = row < rows_active && ok_s;
             // keys j < lim are visible to this row; a full prefix tile needs no
             // mask (rows of other lanes are computed but never stored)
             const int lim = !valid_row ? 0 : (block_tile ? min(nvalid, irow + 1) : nvalid);
@@ -560,17 +581,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (first) {
                 float mt = -INFINITY;
 #pragma unroll 1
-                for (int c = 0; c < kTileKeys; c += 16) {
+                for (int c = 0; c < 32; c += 16) {
                     float v[16];
-                    tmem_ld16(s_addr + c, v);
+                    tmem_ld_half16(s_addr + c, v);
+                    const int key0 = half * 32 + c;
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
-                        mt = fmaxf(mt, c + j < lim ? v[j] * scale : -INFINITY);
+                        mt = fmaxf(mt, key0 + j < lim ? v[j] * scale : -INFINITY);
                 }
-                m_ref = mt;
+                m_ref = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
             }
-            // O and the P buffer of tile k-2 are free once P V of tile k-1 is done
-            if (k >= 1) wait(b_pvdone, (uint32_t)((k - 1) & 1), abort_flag, p.status);
+            // P buffer (k & 1) is free once P V of tile k-2, its last reader, is done
+            // (pvdone[k & 1] completes once per P V of tiles with that parity)
+            if (k >= 2) wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)(((k - 2) >> 1) & 1), abort_flag,
+                             p.status);
             fence_after();
             // P = 2^(s - m) as bf16 into the swizzled P buffer (16 keys = 2 chunks),
             // with the tile max on the side; a second pass only if the max moved
@@ -583,9 +607,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 float mt = -INFINITY;
                 lt = 0.f;
 #pragma unroll 1
-                for (int c = 0; c < kTileKeys; c += 16) {
+                for (int c = 0; c < 32; c += 16) {
                     float v[16];
-                    tmem_ld16(s_addr + c, v);
+                    tmem_ld_half16(s_addr + c, v);
+                    const int key0 = half * 32 + c;
                     uint32_t w[8];
                     if (full_tile) {  // warp-uniform: no masks
                         float vm = v[0];
@@ -602,27 +627,31 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
 #pragma unroll
                         for (int e = 0; e < 8; ++e) {
-                            const float x0 = c + 2 * e < lim ? v[2 * e] * scale : -INFINITY;
-                            const float x1 = c + 2 * e + 1 < lim ? v[2 * e + 1] * scale : -INFINITY;
+                            const float x0 = key0 + 2 * e < lim ? v[2 * e] * scale : -INFINITY;
+                            const float x1 =
+                                key0 + 2 * e + 1 < lim ? v[2 * e + 1] * scale : -INFINITY;
                             mt = fmaxf(mt, fmaxf(x0, x1));
                             const float a = ex2(x0 - mu), b2 = ex2(x1 - mu);
                             lt += a + b2;
                             w[e] = pack_bf16(a, b2);
                         }
                     }
-                    if (owner) {
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                                         p_chunk_addr(pbuf, row, c / 8)),
-                                     "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
-                                     : "memory");
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                                         p_chunk_addr(pbuf, row, c / 8 + 1)),
-                                     "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
-                                     : "memory");
-                    }
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                     p_chunk_addr(pbuf, row, key0 / 8)),
+                                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                 : "memory");
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                     p_chunk_addr(pbuf, row, key0 / 8 + 1)),
+                                 "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                                 : "memory");
                 }
+                mt = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
                 const bool jump = valid_row && !first && mt > m_ref + kRescaleLog2;
                 if (!__any_sync(kFull, jump)) break;
+                // O is stable once P V of tile k-1 is done
+                wait(b_pvdone + 8 * (int)((k - 1) & 1), (uint32_t)(((k - 1) >> 1) & 1), abort_flag,
+                     p.status);
+                fence_after();
                 // the max moved: rescale O and l to the new reference, redo P
                 const float alpha = jump ? ex2(m_ref - mt) : 1.f;  // m_ref -inf gives 0
                 if (jump) {
@@ -665,16 +694,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
             // ---- end of segment: O / l and lse ----
             if (last) {
-                wait(b_pvdone, (uint32_t)(k & 1), abort_flag, p.status);
+                wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1), abort_flag, p.status);
                 fence_after();
                 const long long pair_first = lo + k - ws.t;
                 const bool whole = (seg_first == pair_first) && block_tile;
                 const int pair = ws.b * p.Hkv + ws.h;
                 const size_t slot = (size_t)pair + blockIdx.x;
                 const bool write = owner && row < rows_active;
-                const float inv = l_sum > 0.f ? 1.f / l_sum : 0.f;
-                const float lse =
-                    l_sum > 0.f ? (m_ref + __log2f(l_sum)) * kLn2 : -INFINITY;
+                // the row's sum: this thread's half plus its partner's
+                const float l_row = l_sum + __shfl_xor_sync(kFull, l_sum, 16);
+                const float inv = l_row > 0.f ? 1.f / l_row : 0.f;
+                const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;
                 const int gq = row % p.G;
                 uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
                                           (size_t)ws.h * p.G + gq) * D;
