@@ -40,7 +40,7 @@ FALLBACK_HBM_GBS = 6800.0
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=3000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="das", choices=["das", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
@@ -98,8 +98,10 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            # wait for the first sample so that the timed region is covered
+            self.first = self.proc.stdout.readline()
         except OSError:
             self.proc = None
         return self
@@ -113,6 +115,7 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
                 out, _ = self.proc.communicate()
+            # samples taken while the timed region ran (the first one came before)
             self.lines = [l for l in out.splitlines() if l.strip()]
 
     def summary(self):
@@ -434,22 +437,32 @@ def cpu_baseline(wl, budget_s=12.0):
 
 
 def reference_arm(args):
+    """The fp64 oracle on the host cores, on the same workload, metric and unit.
+    Each step is a bounded sample (one layer call over the first kv heads),
+    sized so that warmup + steps take about a minute in all."""
     rank, world, _ = dist_env()
     if rank != 0:
         return
     from synth import workloads as wlm
     wl = wlm.WORKLOADS[args.workload]
-    heads = sample_heads(wl)
-    sub, K, V, P, T, ins = oracle_sample(wl, heads)
+    if args.layers:
+        wl = wl.replace(layers=args.layers)
+    budget = 60.0 / max(1, args.steps + args.warmup)
+    # time one kv head of one layer, then scale the sample to the budget
+    probe = wl.replace(layers=1)
+    sub, K, V, P, T, ins = oracle_sample(probe, 1)
+    _, t1, _, cores = time_oracle(sub, K, V, P, T, ins[:1], 0.0)
+    heads = int(max(1, min(wl.kv_heads, budget / max(t1, 1e-6))))
+    sub, K, V, P, T, ins = oracle_sample(probe, heads)
     for _ in range(args.warmup):
         time_oracle(sub, K, V, P, T, ins[:1], 0.0)
     per_step = []
     for _ in range(args.steps):
-        gbs, secs, reps, cores = time_oracle(sub, K, V, P, T, ins, 0.0)
+        _, secs, _, cores = time_oracle(sub, K, V, P, T, ins[:1], 0.0)
         per_step.append(secs)
-    nbytes = int(P.astype(np.int64).sum()) * heads * wl.head_dim * 4 * wl.layers
+    nbytes = int(P.astype(np.int64).sum()) * heads * wl.head_dim * 4
     value = nbytes * args.steps / sum(per_step) / 1e9
-    sample = (f"per step: the draft phase ({wl.layers} layers) on kv heads 0..{heads - 1} of "
+    sample = (f"per step: one Mature-V layer call restricted to kv heads 0..{heads - 1} of "
               f"{wl.kv_heads}; fp64 oracle threaded over (sequence, query head)")
     line = {"impl": "reference", "metric": "Mature-V draft-attn prefix-KV GB/s (% of GB300 HBM "
             "peak); draft tokens/s", "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
