@@ -46,6 +46,8 @@ def parse():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-probes", action="store_true",
+                    help="skip the long-prefix draft-phase measurements")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the workload's layer count (smaller profiling captures)")
     ap.add_argument("--compact-depths", action="store_true",
@@ -277,6 +279,10 @@ def gpu_arm(args):
     elif e2e is not None:
         e2e.pop("_seconds")
 
+    probes = None
+    if not args.no_probes:
+        probes = {n: draft_probe(n, dev, 200, 5, peak) for n in ("long", "batched")}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(wl, budget_s=12.0)
@@ -315,7 +321,8 @@ def gpu_arm(args):
                      "frac": round(achieved / peak, 4), "traffic": traffic,
                      "kernel": "attn_kernel (one Mature-V layer call)",
                      "peak_source": f"{peak_kind} HBM copy bandwidth"},
-        "gpu_launches": K_steps * (2 * L * 2 + 2 + 2),
+        "long_prefix_draft": probes,
+        "gpu_launches": K_steps * (2 * L * 2 + 1 + 2),
         "e2e": e2e,
         "cpu_baseline": cpu,
         "clocks": clocks.summary(),
@@ -325,6 +332,65 @@ def gpu_arm(args):
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def draft_probe(name, dev, steps, warmup, peak):
+    """Per-call time of another workload's draft phase, timed like the main
+    one (a CUDA graph of its L layer calls, L2 flushed before every replay).
+    Only the two depth slabs the calls read are stored (depths compacted to
+    key slab 1 and value slab 2): the bytes read are those of the full cache."""
+    import torch
+
+    import paper_2609_34538_gb300 as das
+    from synth import device as sdev
+    from synth import workloads as wlm
+
+    wl = wlm.WORKLOADS[name].replace(depths=2, key_depth=1, value_depth=2)
+    L, B, W = wl.layers, wl.batch, wl.max_block
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        K, V = sdev.build_cache(wl, device=dev)
+        cache = das.DepthKVCache(K, V)
+        pl = torch.from_numpy(wl.prefix_lens()).to(dev)
+        bl = torch.from_numpy(wl.block_lens()).to(dev)
+        ws = das.new_workspace(cache, wl.q_heads, W, device=dev)
+        ins = [sdev.layer_inputs(wl, l, dev) for l in range(L)]
+        outs = [(torch.empty_like(q), torch.empty((B, wl.q_heads, W), dtype=torch.float32,
+                                                  device=dev)) for q, _, _ in ins]
+        flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+    stream.synchronize()
+
+    def phase():
+        for l, (q, kb, vb) in enumerate(ins):
+            das.das_mature_v_attention(cache, l, 1, 2, pl, bl, q, kb, vb, ws, out=outs[l][0],
+                                       lse=outs[l][1], stream=stream)
+
+    with torch.cuda.stream(stream):
+        phase()
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        phase()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(warmup + steps)]
+    for e0, e1 in ev:
+        with torch.cuda.stream(stream):
+            flush.fill_(1)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+    stream.synchronize()
+    ms = [e0.elapsed_time(e1) for e0, e1 in ev[warmup:]]
+    if das.workspace_status(ws) != 0:
+        raise SystemExit(f"bench: {name} draft phase reported a device-side error")
+    nbytes = wl.prefix_bytes_per_layer() * L
+    gbs = nbytes * len(ms) / (sum(ms) / 1e3) / 1e9
+    del K, V, cache, flush
+    torch.cuda.empty_cache()
+    return {"workload": wl.name, "depth_slabs_stored": "2 (the key and value slabs read)",
+            "per_call_us": round(statistics.mean(ms) * 1e3 / L, 2), "gbs": round(gbs, 1),
+            "pct_of_measured_hbm": round(100 * gbs / peak, 1),
+            "pct_of_nominal_8000": round(100 * gbs / 8000.0, 1), "steps": len(ms)}
 
 
 def e2e_arm(args, wl, cache, pl, P0, bl, ws, stream, dev):

@@ -98,14 +98,11 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
 
     // queries: rows of one pair are heads h*G .. h*G+G-1 of every block row i,
     // i.e. a {64, G, max_block, 1} box over [B][max_block][Hq][D]
-    const bool use_tc = true;
     CUtensorMap tq;
-    if (use_tc) {
-        const cuuint64_t q_dims[4] = {(cuuint64_t)D, (cuuint64_t)num_q_heads,
-                                      (cuuint64_t)max_block, (cuuint64_t)c->batch};
-        const cuuint32_t q_box[4] = {64, (cuuint32_t)G, (cuuint32_t)max_block, 1};
-        if (!encode_bf16(&tq, const_cast<void *>(q), 4, q_dims, q_box)) return DAS_ERR_CUDA;
-    }
+    const cuuint64_t q_dims[4] = {(cuuint64_t)D, (cuuint64_t)num_q_heads, (cuuint64_t)max_block,
+                                  (cuuint64_t)c->batch};
+    const cuuint32_t q_box[4] = {64, (cuuint32_t)G, (cuuint32_t)max_block, 1};
+    if (!encode_bf16(&tq, const_cast<void *>(q), 4, q_dims, q_box)) return DAS_ERR_CUDA;
 
     AttnParams p;
     p.prefix_len = prefix_len;
@@ -124,11 +121,10 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
     p.value_slab = (value_depth - 1) * c->layers + layer;
     const double scale = softmax_scale > 0.f ? (double)softmax_scale : 1.0 / sqrt((double)D);
     p.scale_log2 = (float)(scale * 1.4426950408889634);
-    p.num_ctas = use_tc ? attn_tc_grid_size(dev) : attn_grid_size(dev);
+    p.num_ctas = attn_grid_size(dev);
     attn_workspace_layout(workspace, c->batch, c->kv_heads, p.rows_max, D, p.num_ctas, p);
     const cudaError_t e =
-        use_tc ? attn_tc_launch(p, D, tk, tv, tkb, tvb, tq, static_cast<cudaStream_t>(stream))
-               : attn_launch(p, D, tk, tv, tkb, tvb, static_cast<cudaStream_t>(stream));
+        attn_launch(p, D, tk, tv, tkb, tvb, tq, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? DAS_OK : DAS_ERR_CUDA;
 }
 

@@ -1,67 +1,79 @@
-// das_attention.cu -- depth-asynchronous attention (Eqs. 2-3, Sec. 3.2) and the
-// full-depth verify attention (Sec. 3.4) on sm_103a, tensor-core path with
-// mma.sync.
+// das_attention.cu -- depth-asynchronous attention (Eqs. 2-3, Sec. 3.2) and
+// the full-depth verify attention (Sec. 3.4) on the 5th-generation tensor
+// cores of sm_103a (tcgen05, accumulators in tensor memory).
 //
-// Work decomposition.  Each (sequence b, kv head h) pair owns nt_b =
-// ceil(P_b / 64) prefix tiles and one block tile (the draft block's own keys
-// under the causal mask).  All pairs' tiles are laid end to end and the
-// persistent grid of C CTAs takes equal contiguous ranges of that list, so
-// ragged prefix lengths balance by construction.  A CTA's range is cut into
-// segments at pair boundaries.  A segment that covers a whole pair writes the
-// final output.  Otherwise it writes one partial softmax state per query row
-// (O / l and lse) to workspace slot p + c (p = pair index, c = CTA index:
-// unique because both increase along the list).  A second kernel, launched as
-// a programmatic dependent of the first, merges the pairs that were split,
-//     lse = log sum_s exp(lse_s),  O = sum_s exp(lse_s - lse) O_s,
-// one warp per query row with all of the row's partials loaded at once.
+// Work decomposition: every (sequence, kv head) pair owns ceil(P/64) prefix
+// tiles plus one block tile; all pairs' tiles form one list of N tiles, and
+// CTA c of a persistent grid of C CTAs (one per SM) takes the range
+// [c N / C, (c+1) N / C), cut into segments at pair boundaries.  A segment
+// that covers its pair writes the output.  The others write a partial (O / l
+// and the log-sum-exp of their keys) to the workspace, and merge_kernel,
+// launched right after as a programmatic dependent, combines each split
+// pair's partials by log-sum-exp.
 //
-// Inside a CTA: TMA loads of 64-key K and V tiles (128-byte swizzled, two
-// 64-wide panels for D = 128) run STAGES tiles ahead in a ring of shared-
-// memory stages; an mbarrier per stage signals the bytes landed, and the last
-// of the four warps to finish reading a stage refills it (a shared counter,
-// no waiting).  Warps 0-3 compute with mma.sync m16n8k16 (bf16
-// in, fp32 accumulate): S = Q K^T, fp32 online softmax in base 2, O += P V.
-// Query rows of a pair are r = i * G + g (block row i, group member g); 16
-// rows make an m-tile.  With one m-tile the four warps split each tile's keys
-// four ways (KS = 4), with two m-tiles two ways (KS = 2), with three or four
-// m-tiles every warp takes one m-tile and all 64 keys (KS = 1).  Warps that
-// shared an m-tile combine their states through shared memory at the end of
-// the segment.
+// One CTA = four softmax warps + one TMA warp + one MMA warp.
+//   producer (warp 4): TMA loads of 64-key K and V tiles STAGES ahead into a
+//     ring of shared-memory stages, and of each segment's query rows (the
+//     pair's G * max_block rows, ordered i * G + g, which is the order of a
+//     {64, G, max_block} box).
+//   MMA (warp 5, one elected lane issues):
+//       S = Q K^T    tcgen05.mma M=64 N=64 K=D   -> S buffer (k % 2) in TMEM
+//       O += P V     tcgen05.mma M=64 N=D K=64   -> O in TMEM
+//     S of tile k+2 is issued right after P V of tile k, so the tensor core
+//     works ahead while the softmax warps handle the current tile.  A stage is
+//     refilled once the P V that read it has completed.
+//   softmax warps: an M=64 MMA puts row r in TMEM lane 32 (r / 16) + r % 16, so
+//     warp w owns rows 16w..16w+15 and two threads share a row (one per half
+//     of the 64 keys).  They load the row's scores, mask and scale them (base
+//     2), keep a reference max m that only moves when a score exceeds it by
+//     more than 2^8 (then O and l are rescaled in TMEM), write P = 2^(s - m)
+//     as bf16 into a 128-byte-swizzled [64 rows][64 keys] buffer (the K-major
+//     A operand of P V) and accumulate l.  At the end of a segment they read
+//     the O rows from TMEM and write O / l and the lse (or the partial).
+// The kernel is launched as a programmatic dependent of the previous kernel
+// in the stream: barrier set-up and the tensor-memory allocation overlap the
+// previous kernel's tail, and nothing global is read or written before
+// griddepcontrol.wait.  Every wait is bounded (2 s); a time-out sets the
+// status word and stops the CTA's waits.  Tensor memory (256 columns) is freed
+// before the CTA exits.
 #include <cuda_bf16.h>
 
 #include "das_internal.h"
 
 namespace das {
+namespace tc {
 namespace {
 
 constexpr uint32_t kFull = 0xffffffffu;
-constexpr unsigned long long kWaitNs = 2000000000ull;  // 2 s guard on every wait
+constexpr unsigned long long kWaitNs = 2000000000ull;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr int kThreads = kAttnThreads;  // 4 warps
+constexpr int kStages = 4;
+constexpr int kSoftWarps = 4;
+constexpr int kProducerWarp = kSoftWarps;     // TMA loads
+constexpr int kMmaWarp = kSoftWarps + 1;      // tcgen05 MMAs
+constexpr int kThreads = (kSoftWarps + 2) * 32;
+constexpr int kRows = 64;            // M of every MMA (query rows per pair)
+constexpr int kTmemCols = 256;       // S buffers [0, 128), O [128, 128 + D)
+constexpr float kRescaleLog2 = 8.f;  // move the reference max only beyond 2^8
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-
 __device__ __forceinline__ unsigned long long globaltimer() {
     unsigned long long t;
     asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
     return t;
 }
-
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
 }
-
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                  : "memory");
 }
-
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
-
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
@@ -72,13 +84,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-
-// Wait for the phase of `parity` to complete, at most kWaitNs.  On time-out,
-// or if another thread of the CTA already timed out, returns false, raises
-// the CTA's abort flag and the workspace status bit; callers then skip work
-// but keep the CTA's control flow (and its named barriers) intact.
-__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity,
-                                            volatile int *abort_flag, int32_t *status) {
+// Bounded wait; false after 2 s or once another thread of the CTA gave up.
+__device__ __noinline__ bool wait_slow(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                       int32_t *status) {
     const unsigned long long t0 = globaltimer();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
@@ -92,19 +100,17 @@ __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity,
         }
     }
 }
-
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
-                                          int32_t *status) {
+__device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                     int32_t *status) {
 #pragma unroll 1
-    for (int i = 0; i < 16; ++i)
+    for (int i = 0; i < 8; ++i)
         if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    return mbar_wait_slow(bar, parity, abort_flag, status);
+    return wait_slow(bar, parity, abort_flag, status);
 }
 
-__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
-                                            int c0, int c1, int c2, int c3, int c4,
-                                            uint64_t policy) {
+__device__ __forceinline__ void tma_5d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
+                                       int c1, int c2, int c3, int c4, uint64_t policy) {
     asm volatile(
         "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         ".L2::cache_hint [%0], [%1, {%3, %4, %5, %6, %7}], [%2], %8;" ::"r"(dst),
@@ -112,9 +118,8 @@ __device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap *map
         "r"(c4), "l"(policy)
         : "memory");
 }
-
-__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
-                                            int c0, int c1, int c2, int c3) {
+__device__ __forceinline__ void tma_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
+                                       int c1, int c2, int c3) {
     asm volatile(
         "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
@@ -122,27 +127,101 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                        uint32_t &r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
+// ---- tcgen05 ----------------------------------------------------------------
+// Shared-memory matrix descriptor: start, leading / stride byte offsets,
+// descriptor version 1, layout 2 = 128-byte swizzle.
+__device__ __forceinline__ uint64_t sdesc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((addr >> 4) & 0x3FFF) | (uint64_t)((lbo >> 4) & 0x3FFF) << 16 |
+           (uint64_t)((sbo >> 4) & 0x3FFF) << 32 | (uint64_t)1 << 46 | (uint64_t)2 << 61;
 }
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                          uint32_t &r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
+// Instruction descriptor of kind::f16: bf16 A and B, fp32 D, majors, N, M.
+__host__ __device__ constexpr uint32_t idesc(int M, int N, int a_mn_major, int b_mn_major) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn_major << 15) |
+           ((uint32_t)b_mn_major << 16) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
-
-__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
+__device__ __forceinline__ void mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id,
+                                    uint32_t accumulate) {
     asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-        "{%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(id), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// true on exactly one lane of the (converged) warp
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred;
+    asm volatile(
+        "{\n .reg .pred P;\n .reg .b32 R;\n elect.sync R|P, 0xffffffff;\n"
+        " selp.u32 %0, 1, 0, P;\n}\n"
+        : "=r"(pred));
+    return pred != 0;
+}
+// 32 lanes x 32 consecutive 32-bit columns; thread t gets lane (base + t).
+// The load and its wait form one statement, so no use of the registers can
+// be scheduled before the data is there.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+// 16 lanes x 2 halves: thread t < 16 gets lane t, columns [c, c + 16); thread
+// t + 16 gets lane t, columns [c + 32, c + 48).  With M = 64 a warp's rows sit
+// in its first 16 lanes, so two threads share each row.
+__device__ __forceinline__ void tmem_ld_half16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15}, [%16], 32;\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+            taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+        "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+        "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+        "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+        "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+        "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+        "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+        "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ float ex2(float x) {
@@ -150,23 +229,13 @@ __device__ __forceinline__ float ex2(float x) {
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
-
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     uint32_t r;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
 }
 
-// Keep the bf16 halves of `v` whose key index is below `limit`.
-__device__ __forceinline__ uint32_t keep_keys(uint32_t v, int key_lo, int limit) {
-    uint32_t m = (key_lo < limit ? 0x0000ffffu : 0u) | (key_lo + 1 < limit ? 0xffff0000u : 0u);
-    return v & m;
-}
-
-__device__ __forceinline__ void consumers_sync() {
-    asm volatile("bar.sync 1, %0;" ::"n"(kThreads) : "memory");
-}
-
+// ---- tile list ----------------------------------------------------------------
 __device__ __forceinline__ int clamp_prefix(const AttnParams &p, int b) {
     int v = p.prefix_len[b];
     return v < 0 ? 0 : (v > p.capacity ? p.capacity : v);
@@ -176,59 +245,17 @@ __device__ __forceinline__ int clamp_block(const AttnParams &p, int b) {
     return v < 0 ? 0 : (v > p.max_block ? p.max_block : v);
 }
 __device__ __forceinline__ int tiles_of(int P) { return (P + kTileKeys - 1) / kTileKeys + 1; }
-
-// Total tiles N, computed by one warp (all lanes get it).
-__device__ long long total_tiles(const AttnParams &p) {
-    int lane = threadIdx.x & 31;
-    long long acc = 0;
-    for (int b = lane; b < p.B; b += 32) acc += (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv;
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) acc += __shfl_xor_sync(kFull, acc, d);
-    return acc;
-}
-
-// Sequence b whose tiles contain list position x, and the list position of
-// its first tile.  Executed by a whole warp.
-__device__ void locate(const AttnParams &p, long long x, int &b_out, long long &base_out) {
-    int lane = threadIdx.x & 31;
-    long long run = 0;
-    for (int b0 = 0; b0 < p.B; b0 += 32) {
-        int b = b0 + lane;
-        long long v = b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
-        long long inc = v;
-#pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-            long long t = __shfl_up_sync(kFull, inc, d);
-            if (lane >= d) inc += t;
-        }
-        long long total = __shfl_sync(kFull, inc, 31);
-        if (run + total > x) {
-            unsigned m = __ballot_sync(kFull, run + inc > x);
-            int first = __ffs(m) - 1;
-            long long exc = __shfl_sync(kFull, inc - v, first);
-            b_out = b0 + first;
-            base_out = run + exc;
-            return;
-        }
-        run += total;
-    }
-    b_out = p.B;
-    base_out = run;
-}
-
-// Range [c N / C, (c+1) N / C) of CTA c; the CTA whose range holds x.
 __device__ __forceinline__ long long range_lo(int c, long long N, int C) {
     return (long long)c * N / C;
 }
-__device__ __forceinline__ int cta_of(long long x, long long N, int C) {
-    return (int)(((x + 1) * (long long)C - 1) / N);
+// The CTA whose range holds tile t: the largest c with c N / C <= t.
+__device__ __forceinline__ int cta_of(long long t, long long N, int C) {
+    return (int)(((t + 1) * C - 1) / N);
 }
 
-// Position in the tile list: sequence b, kv head h, tile t of nt.
 struct Walk {
     int b, h, t, nt, P, T;
 };
-
 __device__ __forceinline__ void walk_load_seq(const AttnParams &p, Walk &w) {
     if (w.b < p.B) {
         w.P = clamp_prefix(p, w.b);
@@ -236,7 +263,6 @@ __device__ __forceinline__ void walk_load_seq(const AttnParams &p, Walk &w) {
         w.nt = tiles_of(w.P);
     }
 }
-
 __device__ __forceinline__ void walk_next(const AttnParams &p, Walk &w) {
     if (++w.t == w.nt) {
         w.t = 0;
@@ -248,520 +274,525 @@ __device__ __forceinline__ void walk_next(const AttnParams &p, Walk &w) {
     }
 }
 
-template <int D>
-struct Smem {
-    static constexpr int kPanels = D / 64;
-    static constexpr int kTileBytes = kTileKeys * D * 2;  // one of K or V
-    static constexpr int kStageBytes = 2 * kTileBytes;
-};
-
-// Epilogue scratch of the KS > 1 merge: per warp 16 rows x D fp32 values,
-// written into the stage of the segment's last tile (held until the epilogue
-// ends; 4 x 16 x D x 4 bytes is exactly one stage).  Columns are XOR-swizzled
-// by row so that the eight rows a warp writes at once fall in different banks.
-__device__ __forceinline__ int epi_index(int w, int row, int col, int D) {
-    return (w * 16 + row) * D + (col ^ ((row & 7) << 2));
-}
-
-template <int D, int STAGES>
-constexpr int attn_smem_bytes() {
-    return 1024 /* alignment slack */ + STAGES * Smem<D>::kStageBytes +
-           kConsumerWarps * 16 * 2 * 4 /* m, l exchange */ + STAGES * 8 /* mbarriers */ +
-           8 + 4 * STAGES /* flags, arrival counters */;
-}
-
-// Address of (key, 16-byte chunk cg) inside a 128B-swizzled [64 keys][D] tile
-// stored as D/64 panels of 64 rows x 128 bytes.
-__device__ __forceinline__ uint32_t swz(uint32_t tile, int key, int cg) {
-    return tile + ((cg >> 3) << 13) + (key << 7) + ((((cg & 7) ^ (key & 7))) << 4);
-}
-
-// Everything one CTA keeps while walking its range.
-struct Ctx {
-    const AttnParams *p;
-    const CUtensorMap *tm_k, *tm_v, *tm_kb, *tm_vb;
-    uint8_t *stage_base;
-    float *xml;
-    volatile int *abort_flag;
-    int *arrivals;  // [STAGES] count of warp releases of each stage
-    uint32_t full0;
-    long long lo, hi, N;
-    int c;
-    // consumer position
-    Walk w;
-    long long g, k;
-    uint64_t policy;
-};
-
-// Load the tile at walk position wt into stage s (one thread).
-template <int D>
-__device__ __forceinline__ void issue_tile(const Ctx &x, const Walk &wt, int s) {
-    using S = Smem<D>;
-    const uint32_t full = x.full0 + 8 * s;
-    const uint32_t kdst = smem_u32(x.stage_base + s * S::kStageBytes);
-    const uint32_t vdst = kdst + S::kTileBytes;
-    mbar_arrive_expect_tx(full, S::kStageBytes);
-    if (wt.t < wt.nt - 1) {
-        const int tok = wt.t * kTileKeys;
-#pragma unroll
-        for (int dp = 0; dp < S::kPanels; ++dp) {
-            tma_load_5d(kdst + dp * 8192, x.tm_k, full, dp * 64, wt.h, tok, wt.b, x.p->key_slab,
-                        x.policy);
-            tma_load_5d(vdst + dp * 8192, x.tm_v, full, dp * 64, wt.h, tok, wt.b,
-                        x.p->value_slab, x.policy);
-        }
-    } else {
-#pragma unroll
-        for (int dp = 0; dp < S::kPanels; ++dp) {
-            tma_load_4d(kdst + dp * 8192, x.tm_kb, full, dp * 64, wt.h, 0, wt.b);
-            tma_load_4d(vdst + dp * 8192, x.tm_vb, full, dp * 64, wt.h, 0, wt.b);
-        }
-    }
-}
-
-// Called by every warp (lane 0 acts) once it no longer reads stage s, which
-// holds the tile at list position gt (walk wt).  The last of the four warps
-// refills the stage with the tile STAGES positions later, without waiting.
-template <int D, int STAGES>
-__device__ __forceinline__ void release_stage(const Ctx &x, int s, long long gt, Walk wt) {
-    if ((threadIdx.x & 31) != 0) return;
-    // the counter only grows: every fourth arrival is the last of a tile
-    if (atomicAdd(x.arrivals + s, 1) % kConsumerWarps != kConsumerWarps - 1) return;
-    if (gt + STAGES >= x.hi || *x.abort_flag) return;
-#pragma unroll
-    for (int i = 0; i < STAGES; ++i) walk_next(*x.p, wt);
-    // the other warps' generic-proxy reads of this stage precede their
-    // arrivals; order them before the async-proxy (TMA) writes
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    issue_tile<D>(x, wt, s);
-}
-
-__device__ __forceinline__ bool seg_nonempty(int cc, long long N, int C) {
-    return N >= C || range_lo(cc, N, C) != range_lo(cc + 1, N, C);
-}
-
-// Process the tiles of one segment (one pair, from x.g to the pair's block
-// tile or the end of the range) with KS warps sharing each m-tile, then
-// write its result.
-template <int D, int STAGES, int KS>
-__device__ __forceinline__ void run_segment(Ctx &x) {
-    using S = Smem<D>;
-    constexpr int MT = kConsumerWarps / KS;  // m-tiles
-    constexpr int KPW = kTileKeys / KS;      // keys per warp in a tile
-    constexpr int NT8 = KPW / 8;             // 8-key n-tiles per warp
-    constexpr int KSTEPS = D / 16;
-    constexpr int DTILES = D / 8;
-    constexpr bool SPLIT = NT8 <= 4;  // two accumulator sets halve the S chain
-    constexpr int NS2 = SPLIT ? NT8 : 1;
-    const AttnParams &p = *x.p;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int quad_row = lane >> 2, quad_col = (lane & 3) * 2;
-    const int mw = warp % MT, kw = warp / MT;
-    const int key0 = kw * KPW;
-
-    const int sb = x.w.b, sh = x.w.h, snt = x.w.nt, sT = x.w.T;
-    const int rows_active = p.G * sT;
-    const long long pair_first = x.g - x.w.t;
-    const long long seg_first = x.g;
-    const int rowA = mw * 16 + quad_row, rowB = rowA + 8;
-    const int iA = rowA / p.G, iB = rowB / p.G;
-
-    // queries of rows rowA, rowB as m16n8k16 A fragments (0 for invalid rows)
-    uint32_t qa[KSTEPS][4];
-    {
-        const uint16_t *qA = p.q + (((size_t)sb * p.max_block + iA) * p.Hq + (size_t)sh * p.G +
-                                    rowA % p.G) * D;
-        const uint16_t *qB = p.q + (((size_t)sb * p.max_block + iB) * p.Hq + (size_t)sh * p.G +
-                                    rowB % p.G) * D;
-        const bool vA = rowA < rows_active, vB = rowB < rows_active;
-#pragma unroll
-        for (int kk = 0; kk < KSTEPS; ++kk) {
-            const int c0 = kk * 16 + quad_col;
-            qa[kk][0] = vA ? __ldg(reinterpret_cast<const uint32_t *>(qA + c0)) : 0u;
-            qa[kk][1] = vB ? __ldg(reinterpret_cast<const uint32_t *>(qB + c0)) : 0u;
-            qa[kk][2] = vA ? __ldg(reinterpret_cast<const uint32_t *>(qA + c0 + 8)) : 0u;
-            qa[kk][3] = vB ? __ldg(reinterpret_cast<const uint32_t *>(qB + c0 + 8)) : 0u;
-        }
-    }
-    float o[DTILES][4];
-#pragma unroll
-    for (int j = 0; j < DTILES; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
-    float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-    const bool compute = mw * 16 < rows_active;
-
-    bool block_tile;
-    int last_stage = 0;
-    long long last_g = 0;
-    Walk last_w = x.w;
-    do {
-        const int s = (int)(x.k % STAGES);
-        const uint32_t ph = (uint32_t)((x.k / STAGES) & 1);
-        const bool ok = __all_sync(kFull, mbar_wait(x.full0 + 8 * s, ph, x.abort_flag, p.status));
-        block_tile = (x.w.t == snt - 1);
-        const int nvalid = block_tile ? sT : min(kTileKeys, x.w.P - x.w.t * kTileKeys);
-        const uint32_t kt = smem_u32(x.stage_base + s * S::kStageBytes);
-        const uint32_t vt = kt + S::kTileBytes;
-        if (ok && compute) {
-            // ---- S = Q K^T over this warp's keys ----
-            float sc[NT8][4], sc2[NS2][4];
-#pragma unroll
-            for (int j = 0; j < NT8; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
-#pragma unroll
-            for (int j = 0; j < NS2; ++j) sc2[j][0] = sc2[j][1] = sc2[j][2] = sc2[j][3] = 0.f;
-#pragma unroll
-            for (int kk = 0; kk < KSTEPS; ++kk) {
-#pragma unroll
-                for (int jp = 0; jp < NT8 / 2; ++jp) {
-                    const int key = key0 + jp * 16 + (lane & 7) + ((lane >> 4) << 3);
-                    const int cg = 2 * kk + ((lane >> 3) & 1);
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(swz(kt, key, cg), b0, b1, b2, b3);
-                    if (SPLIT && (kk & 1)) {
-                        mma_bf16(sc2[SPLIT ? 2 * jp : 0], qa[kk], b0, b1);
-                        mma_bf16(sc2[SPLIT ? 2 * jp + 1 : 0], qa[kk], b2, b3);
-                    } else {
-                        mma_bf16(sc[2 * jp], qa[kk], b0, b1);
-                        mma_bf16(sc[2 * jp + 1], qa[kk], b2, b3);
-                    }
-                }
-            }
-            // ---- scale, mask, online softmax (base 2) ----
-            float tmax[2] = {-INFINITY, -INFINITY};
-            const bool masked = block_tile || nvalid < key0 + KPW;
-#pragma unroll
-            for (int j = 0; j < NT8; ++j) {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    float v = sc[j][e];
-                    if (SPLIT) v += sc2[SPLIT ? j : 0][e];
-                    v *= p.scale_log2;
-                    if (masked) {
-                        const int key = key0 + j * 8 + quad_col + (e & 1);
-                        bool valid = key < nvalid;
-                        if (block_tile) valid = valid && key <= ((e >> 1) ? iB : iA);
-                        v = valid ? v : -INFINITY;
-                    }
-                    sc[j][e] = v;
-                    tmax[e >> 1] = fmaxf(tmax[e >> 1], v);
-                }
-            }
-            float alpha[2], mu[2];
-#pragma unroll
-            for (int r = 0; r < 2; ++r) {
-                tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(kFull, tmax[r], 1));
-                tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(kFull, tmax[r], 2));
-                const float mn = fmaxf(m_run[r], tmax[r]);
-                mu[r] = mn == -INFINITY ? 0.f : mn;
-                alpha[r] = ex2(m_run[r] - mu[r]);
-                m_run[r] = mn;
-                l_run[r] *= alpha[r];
-            }
-#pragma unroll
-            for (int j = 0; j < DTILES; ++j) {
-                o[j][0] *= alpha[0];
-                o[j][1] *= alpha[0];
-                o[j][2] *= alpha[1];
-                o[j][3] *= alpha[1];
-            }
-#pragma unroll
-            for (int j = 0; j < NT8; ++j) {
-                sc[j][0] = ex2(sc[j][0] - mu[0]);
-                sc[j][1] = ex2(sc[j][1] - mu[0]);
-                sc[j][2] = ex2(sc[j][2] - mu[1]);
-                sc[j][3] = ex2(sc[j][3] - mu[1]);
-                l_run[0] += sc[j][0] + sc[j][1];
-                l_run[1] += sc[j][2] + sc[j][3];
-            }
-            // ---- O += P V ----
-            const bool tail = nvalid < key0 + KPW;
-#pragma unroll
-            for (int kk2 = 0; kk2 < KPW / 16; ++kk2) {
-                const int kb = key0 + kk2 * 16;
-                const uint32_t pa[4] = {pack_bf16(sc[2 * kk2][0], sc[2 * kk2][1]),
-                                        pack_bf16(sc[2 * kk2][2], sc[2 * kk2][3]),
-                                        pack_bf16(sc[2 * kk2 + 1][0], sc[2 * kk2 + 1][1]),
-                                        pack_bf16(sc[2 * kk2 + 1][2], sc[2 * kk2 + 1][3])};
-#pragma unroll
-                for (int dp = 0; dp < DTILES / 2; ++dp) {
-                    const int key = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
-                    const int cg = 2 * dp + (lane >> 4);
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4_t(swz(vt, key, cg), b0, b1, b2, b3);
-                    if (tail) {  // keys past the end may hold anything: zero them
-                        const int k0 = kb + quad_col;
-                        b0 = keep_keys(b0, k0, nvalid);
-                        b1 = keep_keys(b1, k0 + 8, nvalid);
-                        b2 = keep_keys(b2, k0, nvalid);
-                        b3 = keep_keys(b3, k0 + 8, nvalid);
-                    }
-                    mma_bf16(o[2 * dp], pa, b0, b1);
-                    mma_bf16(o[2 * dp + 1], pa, b2, b3);
-                }
-            }
-        }
-        __syncwarp();
-        last_stage = s;
-        last_g = x.g;
-        last_w = x.w;
-        // with KS > 1 the segment's last stage becomes the epilogue scratch:
-        // it is released after the epilogue
-        if (KS == 1 || !(block_tile || x.g + 1 == x.hi)) release_stage<D, STAGES>(x, s, x.g, x.w);
-        ++x.k;
-        ++x.g;
-        walk_next(p, x.w);
-    } while (!block_tile && x.g < x.hi);
-
-    // ------------------------------ segment result ------------------------------
-    const bool whole = (seg_first == pair_first) && block_tile;
-    const int pair = sb * p.Hkv + sh;
-    const size_t slot = (size_t)pair + x.c;
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        l_run[r] += __shfl_xor_sync(kFull, l_run[r], 1);
-        l_run[r] += __shfl_xor_sync(kFull, l_run[r], 2);
-    }
-    if (KS == 1) {
-        // each warp owns its m-tile: write from registers
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            const int row = r == 0 ? rowA : rowB;
-            if (row >= rows_active) continue;
-            const float f = l_run[r] > 0.f ? 1.f / l_run[r] : 0.f;
-            const float lse = l_run[r] > 0.f ? (m_run[r] + __log2f(l_run[r])) * kLn2 : -INFINITY;
-            const int i = row / p.G, g = row % p.G;
-            if (whole) {
-                uint16_t *orow = p.out + (((size_t)sb * p.max_block + i) * p.Hq +
-                                          (size_t)sh * p.G + g) * D;
-#pragma unroll
-                for (int j = 0; j < DTILES; ++j)
-                    *reinterpret_cast<uint32_t *>(orow + j * 8 + quad_col) =
-                        pack_bf16(o[j][2 * r] * f, o[j][2 * r + 1] * f);
-                if ((lane & 3) == 0)
-                    p.lse[((size_t)sb * p.Hq + (size_t)sh * p.G + g) * p.max_block + i] = lse;
-            } else {
-                float *prow = p.part_o + (slot * p.rows_max + row) * D;
-#pragma unroll
-                for (int j = 0; j < DTILES; ++j)
-                    *reinterpret_cast<float2 *>(prow + j * 8 + quad_col) =
-                        make_float2(o[j][2 * r] * f, o[j][2 * r + 1] * f);
-                if ((lane & 3) == 0) p.part_lse[slot * p.rows_max + row] = lse;
-            }
-        }
-    } else {
-        // exchange (m, l) between the KS warps of an m-tile, scale each warp's
-        // O by exp2(m - M) / L into its own region, then sum the regions.
-        // A warp may run ahead by up to STAGES tiles: wait until every warp
-        // has left the previous segment's use of xml and epi.
-        consumers_sync();
-        if ((lane & 3) == 0) {
-            x.xml[(warp * 16 + quad_row) * 2 + 0] = m_run[0];
-            x.xml[(warp * 16 + quad_row) * 2 + 1] = l_run[0];
-            x.xml[(warp * 16 + quad_row + 8) * 2 + 0] = m_run[1];
-            x.xml[(warp * 16 + quad_row + 8) * 2 + 1] = l_run[1];
-        }
-        consumers_sync();
-        float *epi = reinterpret_cast<float *>(x.stage_base + last_stage * S::kStageBytes);
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            const int rr = quad_row + 8 * r;
-            float M = -INFINITY;
-#pragma unroll
-            for (int k2 = 0; k2 < KS; ++k2) M = fmaxf(M, x.xml[((mw + k2 * MT) * 16 + rr) * 2]);
-            const float Mu = M == -INFINITY ? 0.f : M;
-            float L = 0.f;
-#pragma unroll
-            for (int k2 = 0; k2 < KS; ++k2) {
-                const int ww = mw + k2 * MT;
-                L += ex2(x.xml[(ww * 16 + rr) * 2] - Mu) * x.xml[(ww * 16 + rr) * 2 + 1];
-            }
-            const float f = L > 0.f ? ex2(m_run[r] - Mu) / L : 0.f;
-#pragma unroll
-            for (int j = 0; j < DTILES; ++j)
-                *reinterpret_cast<float2 *>(epi + epi_index(warp, rr, j * 8 + quad_col, D)) =
-                    make_float2(o[j][2 * r] * f, o[j][2 * r + 1] * f);
-        }
-        consumers_sync();
-        constexpr int C4 = D / 4;
-        for (int idx = threadIdx.x; idx < MT * 16 * C4; idx += kThreads) {
-            const int row = idx / C4, c4 = idx % C4;
-            if (row >= rows_active) continue;
-            const int mt = row >> 4, rr = row & 15;
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            float M = -INFINITY;
-#pragma unroll
-            for (int k2 = 0; k2 < KS; ++k2) {
-                const int ww = mt + k2 * MT;
-                const float4 v =
-                    *reinterpret_cast<const float4 *>(epi + epi_index(ww, rr, 4 * c4, D));
-                acc.x += v.x;
-                acc.y += v.y;
-                acc.z += v.z;
-                acc.w += v.w;
-                M = fmaxf(M, x.xml[(ww * 16 + rr) * 2]);
-            }
-            const int i = row / p.G, g = row % p.G;
-            float lse = -INFINITY;
-            if (c4 == 0) {
-                const float Mu = M == -INFINITY ? 0.f : M;
-                float L = 0.f;
-#pragma unroll
-                for (int k2 = 0; k2 < KS; ++k2) {
-                    const int ww = mt + k2 * MT;
-                    L += ex2(x.xml[(ww * 16 + rr) * 2] - Mu) * x.xml[(ww * 16 + rr) * 2 + 1];
-                }
-                lse = L > 0.f ? (Mu + __log2f(L)) * kLn2 : -INFINITY;
-            }
-            if (whole) {
-                uint16_t *orow = p.out + (((size_t)sb * p.max_block + i) * p.Hq +
-                                          (size_t)sh * p.G + g) * D;
-                *reinterpret_cast<uint2 *>(orow + 4 * c4) =
-                    make_uint2(pack_bf16(acc.x, acc.y), pack_bf16(acc.z, acc.w));
-                if (c4 == 0)
-                    p.lse[((size_t)sb * p.Hq + (size_t)sh * p.G + g) * p.max_block + i] = lse;
-            } else {
-                *reinterpret_cast<float4 *>(p.part_o + (slot * p.rows_max + row) * D + 4 * c4) =
-                    acc;
-                if (c4 == 0) p.part_lse[slot * p.rows_max + row] = lse;
-            }
-        }
-        release_stage<D, STAGES>(x, last_stage, last_g, last_w);
-    }
-
-    if (whole) {
-        // rows past the block are 0 with lse -inf
-        for (int idx = threadIdx.x; idx < (p.rows_max - rows_active) * (D / 2); idx += kThreads) {
-            const int row = rows_active + idx / (D / 2), col = (idx % (D / 2)) * 2;
-            const int i = row / p.G, g = row % p.G;
-            *reinterpret_cast<uint32_t *>(p.out + (((size_t)sb * p.max_block + i) * p.Hq +
-                                                   (size_t)sh * p.G + g) * D + col) = 0u;
-            if (col == 0)
-                p.lse[((size_t)sb * p.Hq + (size_t)sh * p.G + g) * p.max_block + i] = -INFINITY;
-        }
-        return;
-    }
-}
-
-template <int D, int STAGES>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
-    attn_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                const __grid_constant__ CUtensorMap tm_kb,
-                const __grid_constant__ CUtensorMap tm_vb, const AttnParams p) {
-    using S = Smem<D>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                                ~uintptr_t(1023));
-    Ctx x;
-    x.p = &p;
-    x.tm_k = &tm_k;
-    x.tm_v = &tm_v;
-    x.tm_kb = &tm_kb;
-    x.tm_vb = &tm_vb;
-    x.stage_base = smem;
-    x.xml = reinterpret_cast<float *>(smem + STAGES * S::kStageBytes);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(x.xml + kConsumerWarps * 16 * 2);
-    x.abort_flag = reinterpret_cast<volatile int *>(bars + STAGES);
-    x.arrivals = const_cast<int *>(x.abort_flag) + 2;
-    x.full0 = smem_u32(bars);
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(x.full0 + 8 * s, 1);
-            x.arrivals[s] = 0;
-        }
-        *x.abort_flag = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (threadIdx.x == 32) {
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v)) : "memory");
-    }
-    __syncthreads();
-
-    // This CTA's range [lo, hi) of the tile list and its first position.
-    x.c = blockIdx.x;
+// Range of this CTA and its first position (a whole warp executes this).
+__device__ bool plan(const AttnParams &p, long long &N, long long &lo, long long &hi, Walk &w) {
     const int lane = threadIdx.x & 31;
-    long long base;
-    if (p.B <= 32) {
-        // one load of the lengths per warp; everything else by shuffles
-        const int rawP = lane < p.B ? __ldg(p.prefix_len + lane) : 0;
-        const int rawT = lane < p.B ? __ldg(p.block_len + lane) : 0;
-        const int Pl = rawP < 0 ? 0 : (rawP > p.capacity ? p.capacity : rawP);
-        const int Tl = rawT < 0 ? 0 : (rawT > p.max_block ? p.max_block : rawT);
-        if (x.c == 0 && threadIdx.x < 32 && __any_sync(kFull, rawP != Pl || rawT != Tl) &&
-            lane == 0)
-            atomicOr(p.status, kStatusClamped);
-        const long long v = lane < p.B ? (long long)tiles_of(Pl) * p.Hkv : 0;
+    long long before = 0, total = 0;
+    // pass 1: N
+    for (int b0 = 0; b0 < p.B; b0 += 32) {
+        const int b = b0 + lane;
+        total += b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
+    }
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) total += __shfl_xor_sync(kFull, total, d);
+    N = total;
+    lo = range_lo(blockIdx.x, N, p.num_ctas);
+    hi = range_lo(blockIdx.x + 1, N, p.num_ctas);
+    if (lo >= hi) return false;
+    // pass 2: the sequence holding lo
+    long long run = 0;
+    w.b = p.B;
+    for (int b0 = 0; b0 < p.B; b0 += 32) {
+        const int b = b0 + lane;
+        const long long v = b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
         long long inc = v;
 #pragma unroll
         for (int d = 1; d < 32; d <<= 1) {
             const long long t = __shfl_up_sync(kFull, inc, d);
             if (lane >= d) inc += t;
         }
-        x.N = __shfl_sync(kFull, inc, 31);
-        x.lo = range_lo(x.c, x.N, p.num_ctas);
-        x.hi = range_lo(x.c + 1, x.N, p.num_ctas);
-        if (x.lo >= x.hi) return;
-        const int first = __ffs(__ballot_sync(kFull, inc > x.lo)) - 1;
-        base = __shfl_sync(kFull, inc - v, first);
-        x.w.b = first;
-        x.w.P = __shfl_sync(kFull, Pl, first);
-        x.w.T = __shfl_sync(kFull, Tl, first);
-        x.w.nt = tiles_of(x.w.P);
-    } else {
-        x.N = total_tiles(p);
-        x.lo = range_lo(x.c, x.N, p.num_ctas);
-        x.hi = range_lo(x.c + 1, x.N, p.num_ctas);
-        if (x.c == 0 && threadIdx.x == 0) {
-            for (int b = 0; b < p.B; ++b)
-                if (p.prefix_len[b] != clamp_prefix(p, b) || p.block_len[b] != clamp_block(p, b))
-                    atomicOr(p.status, kStatusClamped);
+        const long long tot = __shfl_sync(kFull, inc, 31);
+        if (run + tot > lo) {
+            const int first = __ffs(__ballot_sync(kFull, run + inc > lo)) - 1;
+            before = run + __shfl_sync(kFull, inc - v, first);
+            w.b = b0 + first;
+            break;
         }
-        if (x.lo >= x.hi) return;
-        locate(p, x.lo, x.w.b, base);
-        x.w.P = x.w.T = x.w.nt = 0;
-        walk_load_seq(p, x.w);
+        run += tot;
     }
-    {
-        const long long off = x.lo - base;
-        x.w.h = (int)(off / x.w.nt);
-        x.w.t = (int)(off % x.w.nt);
-    }
-    x.g = x.lo;
-    x.k = 0;
-    // the merge grid may start loading as SMs free up; it waits for this grid
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(x.policy));
-    if (threadIdx.x == 0) {
-        Walk wt = x.w;
-        for (int i = 0; i < STAGES && x.lo + i < x.hi; ++i) {
-            issue_tile<D>(x, wt, i);
-            walk_next(p, wt);
-        }
-    }
-    while (x.g < x.hi) {
-        const int rows = p.G * x.w.T;
-        if (rows <= 16)
-            run_segment<D, STAGES, 4>(x);
-        else if (rows <= 32)
-            run_segment<D, STAGES, 2>(x);
-        else
-            run_segment<D, STAGES, 1>(x);
-    }
+    walk_load_seq(p, w);
+    const long long off = lo - before;
+    w.h = (int)(off / w.nt);
+    w.t = (int)(off % w.nt);
+    return true;
 }
 
-// Merge the partials of every pair that more than one CTA worked on.  Grid:
-// pairs x ceil(rows_max / 4) CTAs of 4 warps, one warp per query row.
 template <int D>
-__global__ void __launch_bounds__(kThreads) merge_kernel(const AttnParams p) {
-    // partials come from the attention grid this grid depends on
+struct Layout {
+    static constexpr int kPanels = D / 64;
+    static constexpr int kTileBytes = kTileKeys * D * 2;  // K or V of one tile
+    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kQBytes = kPanels * kRows * 128;  // one query buffer
+    static constexpr int kPBytes = kRows * kTileKeys * 2;  // one P buffer
+    static constexpr int kStagesOff = 0;
+    static constexpr int kQOff = kStages * kStageBytes;
+    static constexpr int kPOff = kQOff + 2 * kQBytes;
+    static constexpr int kBarOff = kPOff + 2 * kPBytes;
+    // barriers: full[kStages], empty[kStages], qfull[2], qempty[2], sready[2],
+    // sfree[2], pready[2], pvdone[2], drain
+    static constexpr int kNumBars = 2 * kStages + 13;
+    static constexpr int kMiscOff = kBarOff + kNumBars * 8;
+    static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
+};
+
+// K-major 128B-swizzled address of bf16 element (row, col) of a [64][64] panel
+__device__ __forceinline__ uint32_t p_chunk_addr(uint32_t base, int row, int chunk) {
+    return base + row * 128 + ((chunk ^ (row & 7)) << 4);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ CUtensorMap tm_kb,
+                   const __grid_constant__ CUtensorMap tm_vb,
+                   const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
+    using Lt = Layout<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~uintptr_t(1023));
+    const uint32_t sbase = smem_u32(sm);
+    const uint32_t bars = sbase + Lt::kBarOff;
+    const uint32_t b_full = bars, b_empty = bars + 8 * kStages, b_qfull = b_empty + 8 * kStages,
+                   b_qempty = b_qfull + 16, b_sready = b_qempty + 16, b_sfree = b_sready + 16,
+                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 16;
+    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(sm + Lt::kMiscOff);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Lt::kMiscOff + 4);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+
+    // set-up that touches no global memory: it may overlap the previous
+    // kernel in the stream (programmatic dependent launch)
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(b_full + 8 * s, 1);
+            mbar_init(b_empty + 8 * s, 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(b_qfull + 8 * i, 1);
+            mbar_init(b_qempty + 8 * i, 1);
+            mbar_init(b_sready + 8 * i, 1);
+            mbar_init(b_sfree + 8 * i, kSoftWarps);
+            mbar_init(b_pready + 8 * i, kSoftWarps);
+        }
+        mbar_init(b_pvdone, 1);
+        mbar_init(b_pvdone + 8, 1);
+        mbar_init(b_drain, 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile(
+            "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                smem_u32(const_cast<uint32_t *>(tmem_slot))),
+            "n"(kTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if (warp == kProducerWarp && elect_one()) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_q)) : "memory");
+    }
+    fence_before();
+    __syncthreads();
+    fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    // every input (and the workspace) may be written by the previous kernel
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    const int rblocks = (p.rows_max + kConsumerWarps - 1) / kConsumerWarps;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    if (blockIdx.x == 0 && threadIdx.x == 0)
+        for (int b = 0; b < p.B; ++b)
+            if (p.prefix_len[b] != clamp_prefix(p, b) || p.block_len[b] != clamp_block(p, b))
+                atomicOr(p.status, kStatusClamped);
+    long long N, lo, hi;
+    Walk w0 = {0, 0, 0, 1, 0, 0};
+    // an empty range (only when N < C) runs no loop below
+    const long long ntiles = plan(p, N, lo, hi, w0) ? hi - lo : 0;
+
+    if (warp == kProducerWarp) {
+        // ================================ producer ===============================
+        // Warp-uniform loop; one elected lane issues.  Stage s is reused once
+        // the P V that read it has completed (the MMA warp commits empty[s]);
+        // a query buffer once the last S of the segment before last completed.
+        uint64_t policy;
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+        Walk wl = w0;
+        int qseg = -1;
+        bool ok = true;
+        for (long long j = 0; j < ntiles && ok; ++j) {
+            if (j == 0 || wl.t == 0) {  // the segment's query rows
+                ++qseg;
+                const int qb = qseg & 1;
+                if (qseg >= 2)
+                    ok = ok && wait(b_qempty + 8 * qb, (uint32_t)(((qseg - 2) >> 1) & 1),
+                                    abort_flag, p.status);
+                if (ok && elect_one()) {
+                    const uint32_t full = b_qfull + 8 * qb;
+                    const uint32_t dst = sbase + Lt::kQOff + qb * Lt::kQBytes;
+                    mbar_arrive_expect_tx(full, Lt::kPanels * p.rows_max * 128);
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp)
+                        tma_4d(dst + dp * (kRows * 128), &tm_q, full, dp * 64, wl.h * p.G, 0,
+                               wl.b);
+                }
+            }
+            const int s = (int)(j % kStages);
+            if (j >= kStages)
+                ok = ok && wait(b_empty + 8 * s, (uint32_t)(((j - kStages) / kStages) & 1),
+                                abort_flag, p.status);
+            if (ok && elect_one()) {
+                const uint32_t full = b_full + 8 * s;
+                const uint32_t kdst = sbase + Lt::kStagesOff + s * Lt::kStageBytes;
+                const uint32_t vdst = kdst + Lt::kTileBytes;
+                mbar_arrive_expect_tx(full, Lt::kStageBytes);
+                if (wl.t < wl.nt - 1) {
+                    const int tok = wl.t * kTileKeys;
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                        tma_5d(kdst + dp * 8192, &tm_k, full, dp * 64, wl.h, tok, wl.b,
+                               p.key_slab, policy);
+                        tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
+                               p.value_slab, policy);
+                    }
+                } else {
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                        tma_4d(kdst + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
+                        tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
+                    }
+                }
+            }
+            __syncwarp();
+            walk_next(p, wl);
+        }
+    } else if (warp == kMmaWarp) {
+        // ================================== MMA ==================================
+        const uint32_t id_s = idesc(kRows, kTileKeys, 0, 0);
+        const uint32_t id_pv = idesc(kRows, D, 0, 1);
+        // descriptors are affine in the address: build each base once and add
+        // (byte offset >> 4) for buffers and k-steps
+        const uint64_t dq0 = sdesc(sbase + Lt::kQOff, 16, 1024);
+        const uint64_t dk0 = sdesc(sbase + Lt::kStagesOff, 16, 1024);
+        const uint64_t dv0 = sdesc(sbase + Lt::kStagesOff + Lt::kTileBytes, 8192, 1024);
+        const uint64_t dp0 = sdesc(sbase + Lt::kPOff, 16, 1024);
+        Walk wsn = w0;  // walk of the next S
+        int qseg = -1, qcur = 0;
+        bool ok = true;
+        auto next_s = [&](long long kn) {  // S of tile kn, two tiles ahead of P V
+            if (kn == 0 || wsn.t == 0) {
+                ++qseg;
+                qcur = qseg & 1;
+                ok = ok && wait(b_qfull + 8 * qcur, (uint32_t)((qseg >> 1) & 1), abort_flag,
+                                p.status);
+            }
+            const int s = (int)(kn % kStages);
+            ok = ok && wait(b_full + 8 * s, (uint32_t)((kn / kStages) & 1), abort_flag, p.status);
+            if (kn >= 2)
+                ok = ok && wait(b_sfree + 8 * (int)(kn & 1), (uint32_t)(((kn - 2) >> 1) & 1),
+                                abort_flag, p.status);
+            const bool seg_end = (wsn.t == wsn.nt - 1) || (kn + 1 == ntiles);
+            if (ok) {
+                fence_after();
+                if (elect_one()) {
+                    const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
+                    const uint64_t b0 = dk0 + (uint64_t)((s * Lt::kStageBytes) >> 4);
+                    const uint32_t dS = tmem + (uint32_t)((kn & 1) * kTileKeys);
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        // panel kk / 4, then 16 elements (32 bytes) within the 128-byte row
+                        const uint32_t qoff = ((kk >> 2) * (kRows * 128) + (kk & 3) * 32) >> 4;
+                        const uint32_t koff = ((kk >> 2) * 8192 + (kk & 3) * 32) >> 4;
+                        mma(dS, a0 + qoff, b0 + koff, id_s, kk > 0);
+                    }
+                    mma_commit(b_sready + 8 * (int)(kn & 1));
+                    if (seg_end) mma_commit(b_qempty + 8 * qcur);
+                }
+                __syncwarp();
+            }
+            walk_next(p, wsn);
+        };
+        for (long long kn = 0; kn < 2 && kn < ntiles && ok; ++kn) next_s(kn);
+        Walk wm = w0;  // tile of the next P V
+        for (long long k = 0; k < ntiles && ok; ++k) {
+            const bool first = (k == 0) || (wm.t == 0);
+            ok = ok && wait(b_pready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1), abort_flag,
+                            p.status);
+            if (!ok) break;
+            fence_after();
+            if (elect_one()) {
+                const int s = (int)(k % kStages);
+                const uint64_t a0 = dp0 + (uint64_t)(((k & 1) * Lt::kPBytes) >> 4);
+                const uint64_t b0 = dv0 + (uint64_t)((s * Lt::kStageBytes) >> 4);
+                const uint32_t dO = tmem + 2 * kTileKeys;
+#pragma unroll
+                for (int kk = 0; kk < kTileKeys / 16; ++kk)
+                    mma(dO, a0 + (uint64_t)((kk * 32) >> 4), b0 + (uint64_t)((kk * 2048) >> 4),
+                        id_pv, (!first || kk > 0) ? 1u : 0u);
+                mma_commit(b_pvdone + 8 * (int)(k & 1));
+                mma_commit(b_empty + 8 * s);
+            }
+            __syncwarp();
+            if (k + 2 < ntiles) next_s(k + 2);
+            walk_next(p, wm);
+        }
+        // all MMAs issued here are complete before tensor memory is freed
+        // (only a timed-out run can leave any in flight)
+        if (elect_one()) mma_commit(b_drain);
+        __syncwarp();
+        const unsigned long long t0 = globaltimer();
+        while (!mbar_try_wait(b_drain, 0) && globaltimer() - t0 < kWaitNs) {
+        }
+    } else {
+        // ================================ softmax ================================
+        // thread (warp, lane) handles row 16 warp + lane % 16, keys of its half
+        // (lane / 16) of each tile; the epilogue's O rows are read by lanes < 16
+        const int row = warp * 16 + (lane & 15);
+        const int half = lane >> 4;
+        const bool owner = lane < 16;
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        Walk ws = w0;
+        float m_ref = -INFINITY, l_sum = 0.f;
+        int rows_active = 0, irow = 0;
+        long long seg_first = lo;
+        for (long long k = 0; k < ntiles; ++k) {
+            const bool first = (k == 0) || (ws.t == 0);
+            const bool block_tile = ws.t == ws.nt - 1;
+            const bool last = block_tile || (k + 1 == ntiles);
+            if (first) {
+                m_ref = -INFINITY;
+                l_sum = 0.f;
+                rows_active = p.G * ws.T;
+                irow = row / p.G;
+                seg_first = lo + k;
+            }
+            const int nvalid = block_tile ? ws.T : min(kTileKeys, ws.P - ws.t * kTileKeys);
+            const int s = (int)(k % kStages);
+            // ---- scores: two compact passes over 16-column chunks of S ----
+            const bool ok_s = wait(b_sready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1),
+                                   abort_flag, p.status);
+            fence_after();
+            const uint32_t s_addr = tmem + lane_base + (uint32_t)((k & 1) * kTileKeys);
+            const bool valid_row = row < rows_active && ok_s;
+            // keys j < lim are visible to this row; a full prefix tile needs no
+            // mask (rows of other lanes are computed but never stored)
+            const int lim = !valid_row ? 0 : (block_tile ? min(nvalid, irow + 1) : nvalid);
+            const bool full_tile = !block_tile && nvalid == kTileKeys;
+            const float scale = p.scale_log2;
+            // first tile of a segment: the reference max comes from a max pass
+            if (first) {
+                float mt = -INFINITY;
+#pragma unroll 1
+                for (int c = 0; c < 32; c += 16) {
+                    float v[16];
+                    tmem_ld_half16(s_addr + c, v);
+                    const int key0 = half * 32 + c;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        mt = fmaxf(mt, key0 + j < lim ? v[j] * scale : -INFINITY);
+                }
+                m_ref = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
+            }
+            // P buffer (k & 1) is free once P V of tile k-2, its last reader, is done
+            // (pvdone[k & 1] completes once per P V of tiles with that parity)
+            if (k >= 2) wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)(((k - 2) >> 1) & 1), abort_flag,
+                             p.status);
+            fence_after();
+            // P = 2^(s - m) as bf16 into the swizzled P buffer (16 keys = 2 chunks),
+            // with the tile max on the side; a second pass only if the max moved
+            // beyond the reference by more than 2^8
+            const uint32_t pbuf = sbase + Lt::kPOff + (uint32_t)((k & 1) * Lt::kPBytes);
+            float lt = 0.f;
+#pragma unroll 1
+            for (int pass = 0; pass < 2; ++pass) {
+                const float mu = m_ref == -INFINITY ? 0.f : m_ref;
+                float mt = -INFINITY;
+                lt = 0.f;
+#pragma unroll 1
+                for (int c = 0; c < 32; c += 16) {
+                    float v[16];
+                    tmem_ld_half16(s_addr + c, v);
+                    const int key0 = half * 32 + c;
+                    uint32_t w[8];
+                    if (full_tile) {  // warp-uniform: no masks
+                        float vm = v[0];
+#pragma unroll
+                        for (int j = 1; j < 16; ++j) vm = fmaxf(vm, v[j]);
+                        mt = fmaxf(mt, vm * scale);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const float a = ex2(fmaf(v[2 * e], scale, -mu));
+                            const float b2 = ex2(fmaf(v[2 * e + 1], scale, -mu));
+                            lt += a + b2;
+                            w[e] = pack_bf16(a, b2);
+                        }
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const float x0 = key0 + 2 * e < lim ? v[2 * e] * scale : -INFINITY;
+                            const float x1 =
+                                key0 + 2 * e + 1 < lim ? v[2 * e + 1] * scale : -INFINITY;
+                            mt = fmaxf(mt, fmaxf(x0, x1));
+                            const float a = ex2(x0 - mu), b2 = ex2(x1 - mu);
+                            lt += a + b2;
+                            w[e] = pack_bf16(a, b2);
+                        }
+                    }
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                     p_chunk_addr(pbuf, row, key0 / 8)),
+                                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                 : "memory");
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                     p_chunk_addr(pbuf, row, key0 / 8 + 1)),
+                                 "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                                 : "memory");
+                }
+                mt = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
+                const bool jump = valid_row && !first && mt > m_ref + kRescaleLog2;
+                if (!__any_sync(kFull, jump)) break;
+                // O is stable once P V of tile k-1 is done
+                wait(b_pvdone + 8 * (int)((k - 1) & 1), (uint32_t)(((k - 1) >> 1) & 1), abort_flag,
+                     p.status);
+                fence_after();
+                // the max moved: rescale O and l to the new reference, redo P
+                const float alpha = jump ? ex2(m_ref - mt) : 1.f;  // m_ref -inf gives 0
+                if (jump) {
+                    m_ref = mt;
+                    l_sum *= alpha;
+                }
+#pragma unroll 1
+                for (int c = 0; c < D; c += 32) {
+                    float v[32];
+                    const uint32_t ta = tmem + lane_base + (uint32_t)(2 * kTileKeys + c);
+                    tmem_ld32(ta, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] *= alpha;
+                    tmem_st32(ta, v);
+                }
+            }
+            // S of this tile is no longer read: its buffer may take tile k+2
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_sfree + 8 * (int)(k & 1));
+            l_sum += lt;
+            // keys past the end of the tile may hold anything: zero their V rows
+            if (nvalid < kTileKeys) {
+                const uint32_t vt = sbase + Lt::kStagesOff + s * Lt::kStageBytes + Lt::kTileBytes;
+                const int nzero = (kTileKeys - nvalid) * 8 * Lt::kPanels;  // 16-byte chunks
+                for (int i = threadIdx.x; i < nzero; i += kSoftWarps * 32) {
+                    const int panel = i / ((kTileKeys - nvalid) * 8);
+                    const int rem = i % ((kTileKeys - nvalid) * 8);
+                    const int key = nvalid + rem / 8, chunk = rem % 8;
+                    asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                                     vt + panel * 8192 + key * 128 + (chunk << 4)),
+                                 "r"(0u)
+                                 : "memory");
+                }
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
+
+            // ---- end of segment: O / l and lse ----
+            if (last) {
+                wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1), abort_flag, p.status);
+                fence_after();
+                const long long pair_first = lo + k - ws.t;
+                const bool whole = (seg_first == pair_first) && block_tile;
+                const int pair = ws.b * p.Hkv + ws.h;
+                const size_t slot = (size_t)pair + blockIdx.x;
+                const bool write = owner && row < rows_active;
+                // the row's sum: this thread's half plus its partner's
+                const float l_row = l_sum + __shfl_xor_sync(kFull, l_sum, 16);
+                const float inv = l_row > 0.f ? 1.f / l_row : 0.f;
+                const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;
+                const int gq = row % p.G;
+                uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
+                                          (size_t)ws.h * p.G + gq) * D;
+                float *prow = p.part_o + (slot * p.rows_max + row) * D;
+#pragma unroll 1
+                for (int c = 0; c < D; c += 32) {
+                    float v[32];
+                    tmem_ld32(tmem + lane_base + (uint32_t)(2 * kTileKeys + c), v);
+                    if (write) {
+                        if (whole) {
+#pragma unroll
+                            for (int j = 0; j < 32; j += 8)
+                                *reinterpret_cast<uint4 *>(orow + c + j) =
+                                    make_uint4(pack_bf16(v[j] * inv, v[j + 1] * inv),
+                                               pack_bf16(v[j + 2] * inv, v[j + 3] * inv),
+                                               pack_bf16(v[j + 4] * inv, v[j + 5] * inv),
+                                               pack_bf16(v[j + 6] * inv, v[j + 7] * inv));
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; j += 4)
+                                *reinterpret_cast<float4 *>(prow + c + j) =
+                                    make_float4(v[j] * inv, v[j + 1] * inv, v[j + 2] * inv,
+                                                v[j + 3] * inv);
+                        }
+                    }
+                }
+                if (write) {
+                    if (whole)
+                        p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gq) * p.max_block +
+                              irow] = lse;
+                    else
+                        p.part_lse[slot * p.rows_max + row] = lse;
+                }
+                if (whole) {  // rows past the block: 0 and lse -inf
+                    for (int idx = threadIdx.x; idx < (p.rows_max - rows_active) * (D / 8);
+                         idx += kSoftWarps * 32) {
+                        const int r = rows_active + idx / (D / 8), col = (idx % (D / 8)) * 8;
+                        const int ii = r / p.G, gg = r % p.G;
+                        *reinterpret_cast<uint4 *>(p.out + (((size_t)ws.b * p.max_block + ii) *
+                                                                 p.Hq +
+                                                             (size_t)ws.h * p.G + gg) * D + col) =
+                            make_uint4(0u, 0u, 0u, 0u);
+                        if (col == 0)
+                            p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gg) * p.max_block +
+                                  ii] = -INFINITY;
+                    }
+                }
+                fence_before();
+            }
+            walk_next(p, ws);
+        }
+    }
+    // every MMA was waited on by the control lane and the softmax warps
+    fence_before();
+    __syncthreads();
+    fence_after();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "n"(kTmemCols));
+}
+
+}  // namespace
+
+// ---- split-K merge ------------------------------------------------------------
+// One warp per query row of a split pair; lane l holds columns [VPL l,
+// VPL (l+1)).  With partial s holding O_s / l_s and lse_s for the row:
+//   out = sum_s e^(lse_s - M) O_s / l_s / sum_s e^(lse_s - M),
+//   lse = M + ln sum_s e^(lse_s - M),  M = max_s lse_s,
+// and rows past the block get 0 and lse -inf.  The pair's segments are found
+// from the lengths before griddepcontrol.wait (the attention grid this one
+// depends on started after every kernel that could write them had
+// completed); the partials are read after it, 8 segments' loads in flight.
+constexpr int kMergeWarps = 4;
+
+template <int D>
+__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParams p) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    constexpr int VPL = D / 32;
+    constexpr int kSegs = 8;
+    const int rblocks = (p.rows_max + kMergeWarps - 1) / kMergeWarps;
     const int pair = blockIdx.x / rblocks;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int row = (blockIdx.x % rblocks) * kConsumerWarps + warp;
+    const int row = (blockIdx.x % rblocks) * kMergeWarps + warp;
     const int b = pair / p.Hkv, h = pair % p.Hkv;
     const int C = p.num_ctas;
-    // total tiles N and the list position of this pair's first tile
     long long N = 0, before = 0;
     for (int b0 = 0; b0 < p.B; b0 += 32) {
         const int bb = b0 + lane;
@@ -776,149 +807,138 @@ __global__ void __launch_bounds__(kThreads) merge_kernel(const AttnParams p) {
     }
     const int nt = tiles_of(clamp_prefix(p, b));
     const long long first = before + (long long)h * nt;
-    const int c0 = cta_of(first, N, C), c1 = cta_of(first + nt - 1, N, C);
-    int nseg = c1 - c0 + 1;
-    if (N < C) {
-        nseg = 0;
-        for (int cc = c0; cc <= c1; ++cc) nseg += seg_nonempty(cc, N, C);
-    }
-    if (nseg <= 1 || row >= p.rows_max) return;  // single segment: written directly
+    const int c0 = cta_of(first, N, C);
+    // every nonempty CTA holds a tile when N >= C, so the pair's segments are
+    // those of CTAs c0 .. c1; otherwise each tile is a CTA of its own
+    const int nseg = N >= C ? cta_of(first + nt - 1, N, C) - c0 + 1 : nt;
+    const int rows_active = p.G * clamp_block(p, b);
+
+    // partials come from the attention grid
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (nseg <= 1 || row >= p.rows_max) return;  // a single segment wrote its output
     const int i = row / p.G, g = row % p.G;
-    uint16_t *orow = p.out + (((size_t)b * p.max_block + i) * p.Hq + (size_t)h * p.G + g) * D;
+    uint16_t *orow =
+        p.out + (((size_t)b * p.max_block + i) * p.Hq + (size_t)h * p.G + g) * D + VPL * lane;
     float *lrow = p.lse + ((size_t)b * p.Hq + (size_t)h * p.G + g) * p.max_block + i;
-    constexpr int VPL = D / 32;
-    if (row >= p.G * clamp_block(p, b)) {
+    if (row >= rows_active) {
         if (VPL == 4)
-            *reinterpret_cast<uint2 *>(orow + 4 * lane) = make_uint2(0u, 0u);
+            *reinterpret_cast<uint2 *>(orow) = make_uint2(0u, 0u);
         else
-            *reinterpret_cast<uint32_t *>(orow + 2 * lane) = 0u;
+            *reinterpret_cast<uint32_t *>(orow) = 0u;
         if (lane == 0) *lrow = -INFINITY;
         return;
     }
-    const float *plse = p.part_lse + row;
-    const float *po = p.part_o + (size_t)row * D + VPL * lane;
-    const size_t sstride = (size_t)p.rows_max;  // per slot, in rows
-    float M = -INFINITY;
-    for (int cc = c0 + lane; cc <= c1; cc += 32)
-        if (seg_nonempty(cc, N, C)) M = fmaxf(M, plse[((size_t)pair + cc) * sstride]);
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, d));
-    float L = 0.f;
-    float acc[VPL];
+    float M = -INFINITY, L = 0.f, acc[VPL];
 #pragma unroll
     for (int v = 0; v < VPL; ++v) acc[v] = 0.f;
-    for (int base = c0; base <= c1; base += 32) {
-        const int cc = base + lane;
-        float wl = 0.f;
-        if (cc <= c1 && seg_nonempty(cc, N, C)) wl = __expf(plse[((size_t)pair + cc) * sstride] - M);
-        L += wl;
-        const int n = min(32, c1 - base + 1);
-        int t = 0;
-        for (; t + 8 <= n; t += 8) {
-            float w8[8];
-            float vals[8][VPL];
+#pragma unroll 1
+    for (int s0 = 0; s0 < nseg; s0 += kSegs) {
+        float ls[kSegs], os[kSegs][VPL];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                w8[u] = __shfl_sync(kFull, wl, t + u);
-                const float *src = po + ((size_t)pair + base + t + u) * sstride * D;
+        for (int u = 0; u < kSegs; ++u) {
+            ls[u] = -INFINITY;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v) os[u][v] = 0.f;
+            if (s0 + u < nseg) {
+                const int c = N >= C ? c0 + s0 + u : cta_of(first + s0 + u, N, C);
+                const size_t rs = ((size_t)pair + c) * p.rows_max + row;
+                ls[u] = __ldcg(p.part_lse + rs);
+                const float *src = p.part_o + rs * D + VPL * lane;
                 if (VPL == 4) {
-                    const float4 x4 = *reinterpret_cast<const float4 *>(src);
-                    vals[u][0] = x4.x;
-                    vals[u][1 % VPL] = x4.y;
-                    vals[u][2 % VPL] = x4.z;
-                    vals[u][VPL - 1] = x4.w;
+                    const float4 x = __ldcg(reinterpret_cast<const float4 *>(src));
+                    os[u][0] = x.x;
+                    os[u][1 % VPL] = x.y;
+                    os[u][2 % VPL] = x.z;
+                    os[u][VPL - 1] = x.w;
                 } else {
-                    const float2 x2 = *reinterpret_cast<const float2 *>(src);
-                    vals[u][0] = x2.x;
-                    vals[u][VPL - 1] = x2.y;
+                    const float2 x = __ldcg(reinterpret_cast<const float2 *>(src));
+                    os[u][0] = x.x;
+                    os[u][VPL - 1] = x.y;
                 }
             }
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-                if (w8[u] != 0.f)  // empty CTAs (only when N < C) carry weight 0
-#pragma unroll
-                    for (int v = 0; v < VPL; ++v) acc[v] += w8[u] * vals[u][v];
         }
-        for (; t < n; ++t) {
-            const float wgt = __shfl_sync(kFull, wl, t);
-            if (wgt == 0.f) continue;
-            const float *src = po + ((size_t)pair + base + t) * sstride * D;
+        float mn = M;
 #pragma unroll
-            for (int v = 0; v < VPL; ++v) acc[v] += wgt * src[v];
+        for (int u = 0; u < kSegs; ++u) mn = fmaxf(mn, ls[u]);
+        if (mn == -INFINITY) continue;
+        const float a = __expf(M - mn);  // 0 while M is -inf
+        L *= a;
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) acc[v] *= a;
+#pragma unroll
+        for (int u = 0; u < kSegs; ++u) {
+            const float wgt = __expf(ls[u] - mn);  // 0 for absent segments
+            L += wgt;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v) acc[v] += wgt * os[u][v];
         }
+        M = mn;
     }
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) L += __shfl_xor_sync(kFull, L, d);
-    const float inv = 1.f / L;
+    const float inv = L > 0.f ? 1.f / L : 0.f;
     if (VPL == 4)
-        *reinterpret_cast<uint2 *>(orow + 4 * lane) =
-            make_uint2(pack_bf16(acc[0] * inv, acc[1 % VPL] * inv),
-                       pack_bf16(acc[2 % VPL] * inv, acc[VPL - 1] * inv));
+        *reinterpret_cast<uint2 *>(orow) = make_uint2(pack_bf16(acc[0] * inv, acc[1 % VPL] * inv),
+                                                      pack_bf16(acc[2 % VPL] * inv,
+                                                                acc[VPL - 1] * inv));
     else
-        *reinterpret_cast<uint32_t *>(orow + 2 * lane) = pack_bf16(acc[0] * inv, acc[VPL - 1] * inv);
-    if (lane == 0) *lrow = M + __logf(L);
+        *reinterpret_cast<uint32_t *>(orow) = pack_bf16(acc[0] * inv, acc[VPL - 1] * inv);
+    if (lane == 0) *lrow = L > 0.f ? M + __logf(L) : -INFINITY;
 }
 
 template <int D>
-constexpr int kStages = (D == 128) ? 3 : 6;
-
-template <int D>
-cudaError_t merge_launch_d(const AttnParams &p, cudaStream_t stream);
-
-template <int D>
 cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
-                     const CUtensorMap &tkb, const CUtensorMap &tvb, cudaStream_t stream) {
-    constexpr int ST = kStages<D>;
-    constexpr int smem = attn_smem_bytes<D, ST>();
+                     const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
+                     cudaStream_t stream) {
+    constexpr int smem = Layout<D>::kBytes;
     static bool configured[64] = {false};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 64 && !configured[dev]) {
-        e = cudaFuncSetAttribute(attn_kernel<D, ST>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  smem);
         if (e != cudaSuccess) return e;
         configured[dev] = true;
     }
-    attn_kernel<D, ST><<<p.num_ctas, kThreads, smem, stream>>>(tk, tv, tkb, tvb, p);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    return merge_launch_d<D>(p, stream);
-}
-
-template <int D>
-cudaError_t merge_launch_d(const AttnParams &p, cudaStream_t stream) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(p.B * p.Hkv * ((p.rows_max + kConsumerWarps - 1) / kConsumerWarps)));
+    cfg.gridDim = dim3((unsigned)p.num_ctas);
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, attn_kernel<D>, tk, tv, tkb, tvb, tq, p);
+    if (e != cudaSuccess) return e;
+    cfg.gridDim = dim3((unsigned)((long long)p.B * p.Hkv *
+                                  ((p.rows_max + kMergeWarps - 1) / kMergeWarps)));
+    cfg.blockDim = dim3(kMergeWarps * 32);
+    cfg.dynamicSmemBytes = 0;
     return cudaLaunchKernelEx(&cfg, merge_kernel<D>, p);
 }
 
-}  // namespace
+}  // namespace tc
 
 int attn_grid_size(int device) {
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
         return 0;
-    return sms * kCtasPerSm;
+    return sms;
 }
 
+namespace {
+size_t round256(size_t n) { return (n + 255) & ~size_t(255); }
+}  // namespace
+
+// header | part_o [slots][rows_max][D] | part_lse [slots][rows_max], slots =
+// B * Hkv + C (the slot of a segment is pair + CTA).
 size_t attn_workspace_bytes(int device, int batch, int kv_heads, int rows_max, int head_dim) {
     const int C = attn_grid_size(device);
     if (C <= 0) return 0;
     const size_t slots = (size_t)batch * kv_heads + (size_t)C;
-    size_t bytes = kWorkspaceHeader;
-    bytes += slots * rows_max * head_dim * sizeof(float);
-    bytes = (bytes + 255) & ~size_t(255);
-    bytes += slots * rows_max * sizeof(float);
-    return (bytes + 255) & ~size_t(255);
+    return kWorkspaceHeader + round256(slots * rows_max * head_dim * sizeof(float)) +
+           round256(slots * rows_max * sizeof(float));
 }
 
 void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_max, int head_dim,
@@ -928,22 +948,15 @@ void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_ma
     p.status = reinterpret_cast<int32_t *>(ws);
     size_t off = kWorkspaceHeader;
     p.part_o = reinterpret_cast<float *>(ws + off);
-    off += slots * rows_max * head_dim * sizeof(float);
-    off = (off + 255) & ~size_t(255);
+    off += round256(slots * rows_max * head_dim * sizeof(float));
     p.part_lse = reinterpret_cast<float *>(ws + off);
-}
-
-cudaError_t attn_merge_launch(const AttnParams &p, int head_dim, cudaStream_t stream) {
-    if (head_dim == 128) return merge_launch_d<128>(p, stream);
-    if (head_dim == 64) return merge_launch_d<64>(p, stream);
-    return cudaErrorInvalidValue;
 }
 
 cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
                         const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
-                        const CUtensorMap &tm_vb, cudaStream_t stream) {
-    if (head_dim == 128) return launch_d<128>(p, tm_k, tm_v, tm_kb, tm_vb, stream);
-    if (head_dim == 64) return launch_d<64>(p, tm_k, tm_v, tm_kb, tm_vb, stream);
+                        const CUtensorMap &tm_vb, const CUtensorMap &tm_q, cudaStream_t stream) {
+    if (head_dim == 128) return tc::launch_d<128>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+    if (head_dim == 64) return tc::launch_d<64>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
     return cudaErrorInvalidValue;
 }
 

@@ -1,11 +1,29 @@
 // das_commit.cu -- greedy acceptance and the multi-depth cache commit
 // (Sec. 3.4; App. B.1) on sm_103a.
+//
+// Every kernel here is launched as a programmatic dependent of the previous
+// kernel in the stream: it reads nothing before griddepcontrol.wait, and
+// every CTA executes that wait.
+#include <cooperative_groups.h>
+
 #include "das_internal.h"
+
+namespace cg = cooperative_groups;
 
 namespace das {
 namespace {
 
-constexpr int kArgmaxThreads = 512;
+// ---- greedy acceptance --------------------------------------------------------
+// One cluster of kAcceptCtas CTAs per sequence.  CTA j of the cluster scans
+// slice j of the vocabulary for every row i < W of its sequence and keeps its
+// best (value, index) per row in shared memory; after a cluster barrier CTA 0
+// reads the kAcceptCtas candidates of each row through distributed shared
+// memory, writes target_ids, counts the accepted prefix and writes accepted
+// and next_token.
+constexpr int kAcceptCtas = 8;
+constexpr int kAcceptThreads = 1024;
+constexpr int kAcceptWarps = kAcceptThreads / 32;
+constexpr int kMaxW = 1024;
 
 // (value, index) order of the argmax: larger value wins, equal values go to
 // the smaller index, so the result is the first maximum.
@@ -15,117 +33,192 @@ __device__ __forceinline__ void better(float &bv, int &bi, float v, int i) {
         bi = i;
     }
 }
-
-// One CTA per (sequence, proposal) row: target_ids[b][i] = argmax over vocab.
-__global__ void __launch_bounds__(kArgmaxThreads) argmax_kernel(const float *__restrict__ logits,
-                                                                int vocab,
-                                                                int32_t *__restrict__ target_ids) {
-    const size_t row = blockIdx.x;
-    const float *x = logits + row * (size_t)vocab;
-    float bv = -INFINITY;
-    int bi = 0x7fffffff;
-    const bool vec = (vocab & 3) == 0;
-    if (vec) {
-        const float4 *x4 = reinterpret_cast<const float4 *>(x);
-        const int n4 = vocab >> 2;
-        int j = threadIdx.x;
-        for (; j + 3 * kArgmaxThreads < n4; j += 4 * kArgmaxThreads) {
-            float4 a[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) a[u] = __ldcs(x4 + j + u * kArgmaxThreads);
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int base = 4 * (j + u * kArgmaxThreads);
-                better(bv, bi, a[u].x, base);
-                better(bv, bi, a[u].y, base + 1);
-                better(bv, bi, a[u].z, base + 2);
-                better(bv, bi, a[u].w, base + 3);
-            }
-        }
-        for (; j < n4; j += kArgmaxThreads) {
-            const float4 a = __ldcs(x4 + j);
-            better(bv, bi, a.x, 4 * j);
-            better(bv, bi, a.y, 4 * j + 1);
-            better(bv, bi, a.z, 4 * j + 2);
-            better(bv, bi, a.w, 4 * j + 3);
-        }
-    } else {
-        for (int j = threadIdx.x; j < vocab; j += kArgmaxThreads) better(bv, bi, __ldcs(x + j), j);
-    }
+__device__ __forceinline__ void warp_best(float &bv, int &bi) {
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) {
         const float ov = __shfl_xor_sync(0xffffffffu, bv, d);
         const int oi = __shfl_xor_sync(0xffffffffu, bi, d);
         better(bv, bi, ov, oi);
     }
-    __shared__ float sv[kArgmaxThreads / 32];
-    __shared__ int si[kArgmaxThreads / 32];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) {
-        sv[warp] = bv;
-        si[warp] = bi;
-    }
-    __syncthreads();
-    if (warp == 0) {
-        bv = lane < kArgmaxThreads / 32 ? sv[lane] : -INFINITY;
-        bi = lane < kArgmaxThreads / 32 ? si[lane] : 0x7fffffff;
-#pragma unroll
-        for (int d = 16; d > 0; d >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bv, d);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, d);
-            better(bv, bi, ov, oi);
-        }
-        // A row of -inf only keeps bi at its sentinel: the first index wins.
-        if (lane == 0) target_ids[row] = bi == 0x7fffffff ? 0 : bi;
-    }
 }
 
-// accepted[b] = leading matches; next_token[b] as in Sec. 3.4.
-__global__ void accept_count_kernel(const int32_t *__restrict__ draft,
-                                    const int32_t *__restrict__ target_ids, int B, int W,
-                                    int32_t *__restrict__ accepted, int32_t *__restrict__ next) {
-    for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < B; b += gridDim.x * blockDim.x) {
-        const int32_t *d = draft + (size_t)b * W;
-        const int32_t *t = target_ids + (size_t)b * W;
-        int a = 0;
-        while (a < W && d[a] == t[a]) ++a;
-        accepted[b] = a;
-        next[b] = a < W ? t[a] : d[W - 1];
+struct AcceptSmem {
+    float cand_v[kMaxW];  // this CTA's best per row
+    int cand_i[kMaxW];
+    float warp_v[kAcceptWarps];
+    int warp_i[kAcceptWarps];
+    int target[kMaxW];  // CTA 0: the row argmaxes
+    int first_miss;
+};
+
+// VEC = 4: float4 loads (vocab % 4 == 0 and 16-byte aligned logits), else 1.
+template <int VEC>
+__global__ void __launch_bounds__(kAcceptThreads)
+    accept_kernel(const float *__restrict__ logits, const int32_t *__restrict__ draft, int W,
+                  int vocab, int slice, int32_t *__restrict__ accepted,
+                  int32_t *__restrict__ target_ids, int32_t *__restrict__ next_token) {
+    __shared__ AcceptSmem sm;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    const int b = blockIdx.x / kAcceptCtas;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    // threads per row: the CTA's warps split over min(W, 32) rows at a time
+    int tpr = kAcceptThreads;
+    while (tpr > 32 && tpr * W > kAcceptThreads) tpr >>= 1;
+    const int rows_per_pass = kAcceptThreads / tpr, warps_per_row = tpr / 32;
+    const int lo = min(rank * slice, vocab), hi = min(lo + slice, vocab);
+    const int nvec = (hi - lo) / VEC;  // slice is a multiple of VEC
+    for (int i0 = 0; i0 < W; i0 += rows_per_pass) {
+        const int i = i0 + threadIdx.x / tpr;
+        const int part = threadIdx.x % tpr;
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        if (i < W) {
+            const float *row = logits + ((size_t)b * W + i) * (size_t)vocab + lo;
+            if (VEC == 4) {
+                const float4 *x4 = reinterpret_cast<const float4 *>(row);
+                int j = part;
+                for (; j + 3 * tpr < nvec; j += 4 * tpr) {
+                    float4 a[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) a[u] = __ldcs(x4 + j + u * tpr);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int e = lo + 4 * (j + u * tpr);
+                        better(bv, bi, a[u].x, e);
+                        better(bv, bi, a[u].y, e + 1);
+                        better(bv, bi, a[u].z, e + 2);
+                        better(bv, bi, a[u].w, e + 3);
+                    }
+                }
+                for (; j < nvec; j += tpr) {
+                    const float4 a = __ldcs(x4 + j);
+                    const int e = lo + 4 * j;
+                    better(bv, bi, a.x, e);
+                    better(bv, bi, a.y, e + 1);
+                    better(bv, bi, a.z, e + 2);
+                    better(bv, bi, a.w, e + 3);
+                }
+            } else {
+                int j = part;
+                for (; j + 3 * tpr < nvec; j += 4 * tpr) {
+                    float a[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) a[u] = __ldcs(row + j + u * tpr);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) better(bv, bi, a[u], lo + j + u * tpr);
+                }
+                for (; j < nvec; j += tpr) better(bv, bi, __ldcs(row + j), lo + j);
+            }
+        }
+        warp_best(bv, bi);
+        if (lane == 0) {
+            sm.warp_v[warp] = bv;
+            sm.warp_i[warp] = bi;
+        }
+        __syncthreads();
+        if (threadIdx.x < rows_per_pass && i0 + (int)threadIdx.x < W) {
+            float v = -INFINITY;
+            int x = 0x7fffffff;
+            for (int w = 0; w < warps_per_row; ++w)
+                better(v, x, sm.warp_v[threadIdx.x * warps_per_row + w],
+                       sm.warp_i[threadIdx.x * warps_per_row + w]);
+            sm.cand_v[i0 + threadIdx.x] = v;
+            sm.cand_i[i0 + threadIdx.x] = x;
+        }
+        __syncthreads();
     }
+    cluster.sync();  // every CTA's candidates are in its shared memory
+
+    if (rank == 0) {
+        if (threadIdx.x == 0) sm.first_miss = W;
+        __syncthreads();
+        for (int i = threadIdx.x; i < W; i += kAcceptThreads) {
+            float v = -INFINITY;
+            int x = 0x7fffffff;
+#pragma unroll
+            for (int r = 0; r < kAcceptCtas; ++r) {
+                const AcceptSmem *o = cluster.map_shared_rank(&sm, r);
+                better(v, x, o->cand_v[i], o->cand_i[i]);
+            }
+            // a row of -inf keeps the sentinel: the first index wins
+            const int t = x == 0x7fffffff ? 0 : x;
+            sm.target[i] = t;
+            target_ids[(size_t)b * W + i] = t;
+            if (draft[(size_t)b * W + i] != t) atomicMin(&sm.first_miss, i);
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int a = sm.first_miss;
+            accepted[b] = a;
+            next_token[b] = a < W ? sm.target[a] : draft[(size_t)b * W + W - 1];
+        }
+    }
+    cluster.sync();  // CTA 0 has read the others' shared memory
 }
+
+// ---- commit ---------------------------------------------------------------------
+constexpr int kCopyThreads = 256;
+constexpr int kCopyUnroll = 4;
+constexpr int kCopyChunk = kCopyThreads * kCopyUnroll;  // 16-byte words per CTA and tensor
 
 __device__ __forceinline__ int append_count(int32_t a, int W) {
     if (a < 0) a = 0;
     return a + 1 < W ? a + 1 : W;
 }
 
-// Copy the materialized inputs' K/V of slab (depth, layer, b): blockIdx.x is
-// (depth * layers + layer) * batch + b.  Each 16-byte word is one vector copy.
-__global__ void append_copy_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
-                                   const uint4 *__restrict__ kn, const uint4 *__restrict__ vn,
-                                   const int32_t *__restrict__ accepted,
-                                   const int32_t *__restrict__ prefix_len, int batch, int capacity,
-                                   int W, int row_words) {
-    const int slab = blockIdx.x;
-    const int b = slab % batch;
+// Copy of the materialized inputs' K/V.  CTA x handles chunk x % chunks of
+// slab x / chunks, slab = (depth * layers + layer) * batch + b; each thread
+// moves kCopyUnroll 16-byte words of K and of V, all loads before the stores.
+__global__ void __launch_bounds__(kCopyThreads)
+    append_copy_kernel(uint4 *__restrict__ kc, uint4 *__restrict__ vc,
+                       const uint4 *__restrict__ kn, const uint4 *__restrict__ vn,
+                       const int32_t *__restrict__ accepted,
+                       const int32_t *__restrict__ prefix_len, int batch, int capacity, int W,
+                       int row_words, int chunks) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const size_t slab = blockIdx.x / chunks;
+    const int chunk = blockIdx.x % chunks;
+    const int b = (int)(slab % batch);
     const int n = append_count(accepted[b], W);
     const int p = prefix_len[b];
     if (p < 0 || p + n > capacity) return;  // reported by append_finalize_kernel
-    const size_t words = (size_t)n * row_words;
-    const uint4 *ks = kn + (size_t)slab * W * row_words;
-    const uint4 *vs = vn + (size_t)slab * W * row_words;
-    uint4 *kd = kc + ((size_t)slab * capacity + p) * row_words;
-    uint4 *vd = vc + ((size_t)slab * capacity + p) * row_words;
-    for (size_t i = threadIdx.x; i < words; i += blockDim.x) {
-        kd[i] = __ldcs(ks + i);
-        vd[i] = __ldcs(vs + i);
+    const int words = n * row_words;
+    const int w0 = chunk * kCopyChunk + threadIdx.x;
+    if (chunk * kCopyChunk >= words) return;
+    const uint4 *ks = kn + slab * W * row_words;
+    const uint4 *vs = vn + slab * W * row_words;
+    uint4 *kd = kc + (slab * capacity + p) * row_words;
+    uint4 *vd = vc + (slab * capacity + p) * row_words;
+    uint4 a[kCopyUnroll], c[kCopyUnroll];
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+        const int w = w0 + u * kCopyThreads;
+        if (w < words) {
+            a[u] = __ldcs(ks + w);
+            c[u] = __ldcs(vs + w);
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+        const int w = w0 + u * kCopyThreads;
+        if (w < words) {
+            kd[w] = a[u];
+            vd[w] = c[u];
+        }
     }
 }
 
-// Runs after every copy: grow prefix_len or flag the sequence.
+// Runs once every copy has read prefix_len: grow it or flag the sequence.
 __global__ void append_finalize_kernel(const int32_t *__restrict__ accepted,
                                        int32_t *__restrict__ prefix_len, int batch, int capacity,
                                        int W, int32_t *__restrict__ error_flag) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < batch; b += gridDim.x * blockDim.x) {
         const int n = append_count(accepted[b], W);
         const int p = prefix_len[b];
@@ -137,36 +230,66 @@ __global__ void append_finalize_kernel(const int32_t *__restrict__ accepted,
     }
 }
 
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, unsigned cluster,
+                       cudaStream_t stream, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    int n = 1;
+    if (cluster > 1) {
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = cluster;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        n = 2;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = n;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+}
+
 }  // namespace
 
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream) {
     if (B == 0) return cudaSuccess;
-    argmax_kernel<<<B * W, kArgmaxThreads, 0, stream>>>(logits, vocab, target_ids);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    accept_count_kernel<<<(B + 127) / 128, 128, 0, stream>>>(draft, target_ids, B, W, accepted,
-                                                            next_token);
-    return cudaGetLastError();
+    if (W > kMaxW || B > 0x7fffffff / kAcceptCtas) return cudaErrorInvalidValue;
+    const bool vec = (vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(logits) & 15u) == 0;
+    // slices are whole float4s
+    int slice = (vocab + kAcceptCtas - 1) / kAcceptCtas;
+    slice = (slice + 3) & ~3;
+    const dim3 grid((unsigned)(B * kAcceptCtas)), block(kAcceptThreads);
+    return vec ? launch_pdl(accept_kernel<4>, grid, block, kAcceptCtas, stream, logits, draft, W,
+                            vocab, slice, accepted, target_ids, next_token)
+               : launch_pdl(accept_kernel<1>, grid, block, kAcceptCtas, stream, logits, draft, W,
+                            vocab, slice, accepted, target_ids, next_token);
 }
 
 cudaError_t append_launch(const das_kv_cache &c, const void *k_new, const void *v_new,
                           const int32_t *accepted, int W, int32_t *prefix_len,
                           int32_t *error_flag, cudaStream_t stream) {
     const int row_words = c.kv_heads * c.head_dim * 2 / 16;
-    const int slabs = c.depths * c.layers * c.batch;
+    const long long slabs = (long long)c.depths * c.layers * c.batch;
     if (slabs == 0) return cudaSuccess;
-    append_copy_kernel<<<slabs, 256, 0, stream>>>(
-        static_cast<uint4 *>(c.k), static_cast<uint4 *>(c.v), static_cast<const uint4 *>(k_new),
-        static_cast<const uint4 *>(v_new), accepted, prefix_len, c.batch, c.capacity, W,
-        row_words);
-    cudaError_t e = cudaGetLastError();
+    const long long words = (long long)W * row_words;
+    if (words > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const int chunks = (int)((words + kCopyChunk - 1) / kCopyChunk);
+    if (slabs * chunks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    cudaError_t e = launch_pdl(append_copy_kernel, dim3((unsigned)(slabs * chunks)),
+                               dim3(kCopyThreads), 1, stream, static_cast<uint4 *>(c.k),
+                               static_cast<uint4 *>(c.v), static_cast<const uint4 *>(k_new),
+                               static_cast<const uint4 *>(v_new), accepted,
+                               static_cast<const int32_t *>(prefix_len), c.batch, c.capacity, W,
+                               row_words, chunks);
     if (e != cudaSuccess) return e;
-    append_finalize_kernel<<<(c.batch + 127) / 128, 128, 0, stream>>>(accepted, prefix_len,
-                                                                      c.batch, c.capacity, W,
-                                                                      error_flag);
-    return cudaGetLastError();
+    return launch_pdl(append_finalize_kernel, dim3((unsigned)((c.batch + 127) / 128)), dim3(128),
+                      1, stream, accepted, prefix_len, c.batch, c.capacity, W, error_flag);
 }
 
 }  // namespace das

@@ -15,9 +15,6 @@ namespace das {
 // tile for the draft block's own keys.
 constexpr int kTileKeys = 64;
 constexpr int kMaxRows = 64;          // G * max_block handled by one pair
-constexpr int kConsumerWarps = 4;
-constexpr int kAttnThreads = kConsumerWarps * 32;
-constexpr int kCtasPerSm = 2;
 constexpr size_t kWorkspaceHeader = 256;
 
 // Bits of the workspace status word.
@@ -39,7 +36,8 @@ struct AttnParams {
     int num_ctas;
 };
 
-// Number of CTAs the attention kernel launches on `device` (a persistent grid).
+// Number of CTAs the attention kernel launches on `device` (a persistent
+// grid, one CTA per SM).
 int attn_grid_size(int device);
 size_t attn_workspace_bytes(int device, int batch, int kv_heads, int rows_max, int head_dim);
 // Carve a workspace into status word and partials (sets p.status, p.part_o,
@@ -47,22 +45,12 @@ size_t attn_workspace_bytes(int device, int batch, int kv_heads, int rows_max, i
 void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_max, int head_dim,
                            int num_ctas, AttnParams &p);
 
-// Launch the split-K attention kernel and its merge (a programmatic
-// dependent launch) on `stream`.
+// Launch the tcgen05 attention kernel and its split-K merge on `stream`, each
+// a programmatic dependent of the kernel before it; tm_q maps the queries
+// [B][max_block][Hq][D] with a {64, G, max_block, 1} box.
 cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
                         const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
-                        const CUtensorMap &tm_vb, cudaStream_t stream);
-
-// The merge of split pairs alone (a programmatic dependent launch).
-cudaError_t attn_merge_launch(const AttnParams &p, int head_dim, cudaStream_t stream);
-
-// The tcgen05 attention kernel (one CTA per SM) and its merge on `stream`;
-// tm_q maps the queries [B][max_block][Hq][D] with a {64, G, max_block, 1} box.
-int attn_tc_grid_size(int device);
-cudaError_t attn_tc_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
-                           const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
-                           const CUtensorMap &tm_vb, const CUtensorMap &tm_q,
-                           cudaStream_t stream);
+                        const CUtensorMap &tm_vb, const CUtensorMap &tm_q, cudaStream_t stream);
 
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,

@@ -6,7 +6,7 @@ import pytest
 import torch
 
 from synth import workloads as wl_mod
-from tests.gpu_util import dev_bf16, dev_i32, run_small
+from tests.gpu_util import assert_close, dev_bf16, dev_i32, run_small
 
 pytestmark = pytest.mark.gpu
 
@@ -129,6 +129,33 @@ def test_deterministic_and_graph_capturable():
     g.replay()
     torch.cuda.synchronize()
     assert torch.equal(o1, o3) and torch.equal(l1, l3)
+
+
+def test_workspace_reused_by_back_to_back_calls():
+    """Calls enqueued back to back on one workspace (each kernel a programmatic
+    dependent of the one before): every result matches the oracle."""
+    import oracle
+    import paper_2609_34538_gb300 as das
+    wl = small(batch=2, q_heads=8, kv_heads=2, prefix=(3000, 3000), block=(8,))
+    K, V = wl_mod.gen_cache(wl, depths=[2, 8])
+    cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+    ws = das.new_workspace(cache, 8, 8)
+    cases = [(0, [3000, 2900], [8, 5]), (1, [64, 0], [8, 8]), (0, [1, 2999], [3, 8]),
+             (1, [3000, 3000], [8, 8]), (1, [0, 0], [1, 8])]
+    results = []
+    for layer, pl, bl in cases:
+        q = wl_mod.gen_q(wl, layer)
+        kb, vb = wl_mod.gen_block_kv(wl, layer)
+        out, lse = das.das_mature_v_attention(cache, layer, 2, 8, dev_i32(pl), dev_i32(bl),
+                                              dev_bf16(q), dev_bf16(kb), dev_bf16(vb), ws)
+        results.append((layer, pl, bl, q, kb, vb, out, lse))
+    torch.cuda.synchronize()
+    for layer, pl, bl, q, kb, vb, out, lse in results:
+        ref_o, ref_l = oracle.attention(K, V, layer, 2, 8, np.asarray(pl, np.int32),
+                                        np.asarray(bl, np.int32), q, kb, vb)
+        assert_close(out.float().cpu().numpy(), ref_o, lse.cpu().numpy(), ref_l,
+                     where=f"[layer {layer} prefix {pl} block {bl}]")
+    assert das.workspace_status(ws) == 0
 
 
 def test_host_errors_raise():

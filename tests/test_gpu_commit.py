@@ -34,7 +34,8 @@ def test_accept_verify_workload():
     assert np.array_equal(acc, a_star)
 
 
-@pytest.mark.parametrize("B,W,V", [(1, 1, 2), (3, 5, 1001), (2, 16, 7), (4, 32, 50257), (1, 3, 4)])
+@pytest.mark.parametrize("B,W,V", [(1, 1, 2), (3, 5, 1001), (2, 16, 7), (4, 32, 50257), (1, 3, 4),
+                                   (2, 100, 3001), (1, 1024, 64), (5, 8, 32000), (1, 2, 131072)])
 def test_accept_shapes(B, W, V):
     a_star, draft, logits = synth.accept_inputs(B * 100 + W, B, W, V)
     check_accept(logits, draft)
