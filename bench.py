@@ -319,7 +319,7 @@ def gpu_arm(args):
         "verify_gbs": round(verify_bytes * K_steps / (sum(verify_ms) / 1e3) / 1e9, 1),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": traffic,
-                     "kernel": "attn_kernel (one Mature-V layer call)",
+                     "kernel": "attn_kernel + merge_kernel (one Mature-V layer call)",
                      "peak_source": f"{peak_kind} HBM copy bandwidth"},
         "long_prefix_draft": probes,
         "gpu_launches": K_steps * (2 * L * 2 + 1 + 2),
