@@ -11,6 +11,8 @@ ABI in include/das.h:
     das_verify_attention    full-depth verify attention (Sec. 3.4, Eq. 7)
     das_greedy_accept       greedy acceptance (Sec. 3.4)
     das_kv_append           commit of accepted K/V at every depth (App. B.1)
+    AttentionCall           the attention calls with arguments checked once, for
+                            loops that call with the same tensors every step
 
 If libdas.so is missing the import fails: there is no fallback.
 """
@@ -75,11 +77,11 @@ def _check(code, what):
 
 def _stream(stream):
     s = torch.cuda.current_stream() if stream is None else stream
-    return ctypes.c_void_p(s.cuda_stream)
+    return s.cuda_stream
 
 
 def _ptr(t):
-    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+    return t.data_ptr() if t is not None else 0
 
 
 def _need(t, dtype, name, ndim=None):
@@ -209,6 +211,44 @@ def das_verify_attention(cache, layer, depth, prefix_len, block_len, q, k_blk, v
         _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale), _ptr(out), _ptr(lse),
         _ptr(workspace), workspace.numel(), _stream(stream)), "das_verify_attention")
     return out, lse
+
+
+class AttentionCall:
+    """Attention calls with fixed arguments, checked once.
+
+    A serving loop calls attention with the same cache, lengths, inputs,
+    outputs and workspace every step.  This object checks them when it is
+    built and keeps their marshalled pointers, so each call below is a single
+    C call.  The tensors must stay alive, in place and unchanged in shape
+    while the object is used (their contents may change between calls).
+
+        call = AttentionCall(cache, prefix_len, block_len, q, k_blk, v_blk, ws)
+        out, lse = call.mature_v(layer, key_depth, value_depth, stream)
+        out, lse = call.verify(layer, depth, stream)
+    """
+
+    def __init__(self, cache, prefix_len, block_len, q, k_blk, v_blk, workspace, out=None,
+                 lse=None, softmax_scale=0.0):
+        T, Hq, out, lse = _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out,
+                                          lse, workspace)
+        self.cache, self.out, self.lse = cache, out, lse
+        self._keep = (prefix_len, block_len, q, k_blk, v_blk, workspace)
+        self._desc = ctypes.byref(cache.desc)
+        self._args = (_ptr(prefix_len), _ptr(block_len), T, _ptr(q), _ptr(k_blk), _ptr(v_blk),
+                      Hq, float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
+                      workspace.numel())
+
+    def mature_v(self, layer, key_depth, value_depth, stream=None):
+        """das_mature_v_attention (Eqs. 2-3) with this object's arguments."""
+        _check(LIB.das_mature_v_attention(self._desc, layer, key_depth, value_depth, *self._args,
+                                          _stream(stream)), "das_mature_v_attention")
+        return self.out, self.lse
+
+    def verify(self, layer, depth, stream=None):
+        """das_verify_attention (Sec. 3.4) with this object's arguments."""
+        _check(LIB.das_verify_attention(self._desc, layer, depth, *self._args, _stream(stream)),
+               "das_verify_attention")
+        return self.out, self.lse
 
 
 def das_greedy_accept(logits, draft_ids, accepted=None, target_ids=None, next_token=None,

@@ -31,8 +31,8 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 // bf16 tensor map over `rank` dims (innermost first) with 128-byte swizzle;
 // the default box {64, 1, 64, 1, 1} is 64 positions x 64 head_dim elements.
-bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
-                 const cuuint32_t *box_in = nullptr) {
+bool encode_bf16_uncached(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
+                          const cuuint32_t *box) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t strides[4];
@@ -41,14 +41,77 @@ bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
         s *= dims[i];
         strides[i] = s;
     }
-    cuuint32_t box[5] = {64, 1, 64, 1, 1};
-    if (box_in)
-        for (int i = 0; i < rank; ++i) box[i] = box_in[i];
     cuuint32_t estr[5] = {1, 1, 1, 1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, base, dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Encoded maps are kept in a small direct-mapped table keyed by everything
+// the encoding depends on (address, rank, extents, box): a serving loop calls
+// with the same buffers every step, and an encode costs about as much host
+// time as a launch.  A hit returns a copy of the very descriptor an encode
+// would produce, so the table never changes a result.
+struct MapKey {
+    void *base;
+    int rank;
+    cuuint64_t dims[5];
+    cuuint32_t box[5];
+};
+struct MapSlot {
+    bool used;
+    MapKey key;
+    CUtensorMap map;
+};
+constexpr int kMapSlots = 256;
+std::mutex g_map_mu;
+MapSlot g_maps[kMapSlots];
+
+bool same_key(const MapKey &a, const MapKey &b) {
+    if (a.base != b.base || a.rank != b.rank) return false;
+    for (int i = 0; i < a.rank; ++i)
+        if (a.dims[i] != b.dims[i] || a.box[i] != b.box[i]) return false;
+    return true;
+}
+
+bool encode_bf16(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
+                 const cuuint32_t *box_in = nullptr) {
+    MapKey key = {};
+    key.base = base;
+    key.rank = rank;
+    const cuuint32_t box_default[5] = {64, 1, 64, 1, 1};
+    for (int i = 0; i < rank; ++i) {
+        key.dims[i] = dims[i];
+        key.box[i] = box_in ? box_in[i] : box_default[i];
+    }
+    uint64_t h = 1469598103934665603ull;  // FNV-1a over the key's fields
+    auto mix = [&h](uint64_t v) {
+        for (int i = 0; i < 8; ++i) {
+            h ^= (v >> (8 * i)) & 0xffu;
+            h *= 1099511628211ull;
+        }
+    };
+    mix(reinterpret_cast<uintptr_t>(base));
+    mix((uint64_t)rank);
+    for (int i = 0; i < rank; ++i) {
+        mix(key.dims[i]);
+        mix(key.box[i]);
+    }
+    MapSlot &slot = g_maps[h % kMapSlots];
+    {
+        std::lock_guard<std::mutex> lock(g_map_mu);
+        if (slot.used && same_key(slot.key, key)) {
+            *m = slot.map;
+            return true;
+        }
+    }
+    if (!encode_bf16_uncached(m, base, rank, key.dims, key.box)) return false;
+    std::lock_guard<std::mutex> lock(g_map_mu);
+    slot.used = true;
+    slot.key = key;
+    slot.map = *m;
+    return true;
 }
 
 bool cache_ok(const das_kv_cache *c) {

@@ -38,6 +38,8 @@
 // before the CTA exits.
 #include <cuda_bf16.h>
 
+#include <atomic>
+
 #include "das_internal.h"
 
 namespace das {
@@ -204,6 +206,61 @@ __device__ __forceinline__ void tmem_ld_half16(uint32_t taddr, float (&v)[16]) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
 }
+// The O row of the calling thread's half: with M = 64, thread t < 16 of a warp
+// gets TMEM lane t, columns [64 g, 64 g + 32) for g < D / 64, and thread t + 16
+// the same lane, columns [64 g + 32, 64 g + 64).  All loads are issued before
+// the single wait, so the epilogue pays one TMEM round trip.
+template <int D>
+__device__ __forceinline__ void tmem_ld_orow(uint32_t taddr, float (&v)[D / 2]);
+template <>
+__device__ __forceinline__ void tmem_ld_orow<128>(uint32_t taddr, float (&v)[64]) {
+    uint32_t r[64];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%64], 32;\n"
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,"
+        "%27,%28,%29,%30,%31}, [%65], 32;\n"
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,"
+        "%43,%44,%45,%46,%47}, [%66], 32;\n"
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,"
+        "%59,%60,%61,%62,%63}, [%67], 32;\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]),
+          "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]),
+          "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]),
+          "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]),
+          "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]),
+          "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+        : "r"(taddr), "r"(taddr + 16), "r"(taddr + 64), "r"(taddr + 80)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 64; ++j) v[j] = __uint_as_float(r[j]);
+}
+template <>
+__device__ __forceinline__ void tmem_ld_orow<64>(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%32], 32;\n"
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,"
+        "%27,%28,%29,%30,%31}, [%33], 32;\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr), "r"(taddr + 16)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
@@ -245,13 +302,6 @@ __device__ __forceinline__ int clamp_block(const AttnParams &p, int b) {
     return v < 0 ? 0 : (v > p.max_block ? p.max_block : v);
 }
 __device__ __forceinline__ int tiles_of(int P) { return (P + kTileKeys - 1) / kTileKeys + 1; }
-__device__ __forceinline__ long long range_lo(int c, long long N, int C) {
-    return (long long)c * N / C;
-}
-// The CTA whose range holds tile t: the largest c with c N / C <= t.
-__device__ __forceinline__ int cta_of(long long t, long long N, int C) {
-    return (int)(((t + 1) * C - 1) / N);
-}
 
 struct Walk {
     int b, h, t, nt, P, T;
@@ -274,47 +324,129 @@ __device__ __forceinline__ void walk_next(const AttnParams &p, Walk &w) {
     }
 }
 
-// Range of this CTA and its first position (a whole warp executes this).
-__device__ bool plan(const AttnParams &p, long long &N, long long &lo, long long &hi, Walk &w) {
+// Extra weight of a pair's block tile when the list is split.  Ending one
+// segment and starting the next (the mostly empty block tile holding a
+// pipeline slot, the partial write, the first tile's max pass) costs a CTA
+// more than one tile's time.  With few pairs per CTA (at least 4 CTAs per
+// pair) the CTAs whose range holds a block tile are a minority that finishes
+// last, so they take one tile fewer; with many pairs most ranges hold one
+// and the weight only moves work around (measured on the decode, long and
+// batched workloads).
+constexpr int kBlockWeight = 1;
+constexpr int kCtasPerPairForWeight = 4;
+
+// The split of the tile list: tile x of pair q has weighted position
+// x + beta q; CTA c takes the tiles whose weighted position lies in
+// [c W / C, (c+1) W / C).  beta = kBlockWeight if there are at least
+// kCtasPerPairForWeight CTAs per pair and W >= (2 + beta) C (which leaves no
+// CTA empty: weighted positions are at most 1 + beta apart), else 0.
+struct Split {
+    long long N;  // tiles
+    long long W;  // N + beta * pairs
+    int beta;
+};
+
+// The split, given the total tile count.
+__device__ __forceinline__ Split split_from_total(const AttnParams &p, long long total) {
+    const long long pairs = (long long)p.B * p.Hkv;
+    Split sp;
+    sp.N = total;
+    sp.beta = pairs * kCtasPerPairForWeight <= p.num_ctas &&
+                      total + kBlockWeight * pairs >= (long long)(2 + kBlockWeight) * p.num_ctas
+                  ? kBlockWeight
+                  : 0;
+    sp.W = total + sp.beta * pairs;
+    return sp;
+}
+
+// Tiles of one pair of sequence b (0 past the batch); at most 2^25, so sums
+// over 32 sequences fit in 32 bits.
+__device__ __forceinline__ int seq_tiles(const AttnParams &p, int b) {
+    return b < p.B ? tiles_of(clamp_prefix(p, b)) : 0;
+}
+
+__device__ Split split_of(const AttnParams &p) {  // whole warp
     const int lane = threadIdx.x & 31;
-    long long before = 0, total = 0;
-    // pass 1: N
+    long long total = 0;
+    for (int b0 = 0; b0 < p.B; b0 += 32)
+        total += (long long)__reduce_add_sync(kFull, (unsigned)seq_tiles(p, b0 + lane)) * p.Hkv;
+    return split_from_total(p, total);
+}
+
+// The CTA whose weighted range holds weighted position q.
+__device__ __forceinline__ int cta_of_w(long long q, const Split &sp, int C) {
+    return (int)(((q + 1) * C - 1) / sp.W);
+}
+
+// Range [lo, hi) of this CTA and the walk state of its first tile (a whole
+// warp executes this).  One pass over the sequences: a 32-bit inclusive scan
+// of the per-pair tile counts gives, for sequence b of a chunk, both the
+// tiles and the weighted positions before it; the tiles at the weighted
+// positions c W / C and (c+1) W / C are located in the same pass.
+__device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w) {
+    const int lane = threadIdx.x & 31;
+    const Split sp = split_of(p);
+    const long long lw = (long long)blockIdx.x * sp.W / p.num_ctas;
+    const long long hw = ((long long)blockIdx.x + 1) * sp.W / p.num_ctas;
+    lo = hi = sp.N;
+    bool have_lo = false;
+    long long run_w = 0, run_t = 0;  // weighted positions / tiles before the chunk
     for (int b0 = 0; b0 < p.B; b0 += 32) {
-        const int b = b0 + lane;
-        total += b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
-    }
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) total += __shfl_xor_sync(kFull, total, d);
-    N = total;
-    lo = range_lo(blockIdx.x, N, p.num_ctas);
-    hi = range_lo(blockIdx.x + 1, N, p.num_ctas);
-    if (lo >= hi) return false;
-    // pass 2: the sequence holding lo
-    long long run = 0;
-    w.b = p.B;
-    for (int b0 = 0; b0 < p.B; b0 += 32) {
-        const int b = b0 + lane;
-        const long long v = b < p.B ? (long long)tiles_of(clamp_prefix(p, b)) * p.Hkv : 0;
-        long long inc = v;
+        const int nt = seq_tiles(p, b0 + lane);
+        int inc = nt;  // inclusive scan over the chunk
 #pragma unroll
         for (int d = 1; d < 32; d <<= 1) {
-            const long long t = __shfl_up_sync(kFull, inc, d);
-            if (lane >= d) inc += t;
+            const int u = __shfl_up_sync(kFull, inc, d);
+            if (lane >= d) inc += u;
         }
-        const long long tot = __shfl_sync(kFull, inc, 31);
-        if (run + tot > lo) {
-            const int first = __ffs(__ballot_sync(kFull, run + inc > lo)) - 1;
-            before = run + __shfl_sync(kFull, inc - v, first);
-            w.b = b0 + first;
-            break;
+        const int nseq = min(32, p.B - b0);
+        // weighted position after this lane's sequence
+        const long long after_w =
+            run_w + ((long long)inc + (long long)sp.beta * min(lane + 1, nseq)) * p.Hkv;
+        // tile x at weighted position q, q inside sequence f of this chunk
+        auto locate = [&](long long q, int f, Walk *wk) {
+            const int ntf = __shfl_sync(kFull, nt, f);
+            const int excl = __shfl_sync(kFull, inc, f) - ntf;
+            const long long seq_w = run_w + ((long long)excl + (long long)sp.beta * f) * p.Hkv;
+            const long long seq_t = run_t + (long long)excl * p.Hkv;
+            const long long off = q - seq_w;
+            int h = (int)(off / (ntf + sp.beta));
+            int t = (int)(off % (ntf + sp.beta));
+            if (t >= ntf) {  // inside a block tile's extra weight: the next pair
+                t = 0;
+                ++h;
+            }
+            if (wk) {
+                wk->b = b0 + f;
+                wk->h = h;
+                wk->t = t;
+                walk_load_seq(p, *wk);
+                if (wk->h == p.Hkv) {
+                    wk->h = 0;
+                    ++wk->b;
+                    walk_load_seq(p, *wk);
+                }
+            }
+            return seq_t + (long long)h * ntf + t;
+        };
+        if (!have_lo) {
+            const unsigned m = __ballot_sync(kFull, after_w > lw);
+            if (m) {
+                lo = locate(lw, __ffs(m) - 1, &w);
+                have_lo = true;
+            }
         }
-        run += tot;
+        if (have_lo) {
+            const unsigned m = __ballot_sync(kFull, after_w > hw);
+            if (m) {
+                hi = locate(hw, __ffs(m) - 1, nullptr);
+                break;
+            }
+        }
+        run_w += ((long long)__shfl_sync(kFull, inc, 31) + (long long)sp.beta * nseq) * p.Hkv;
+        run_t += (long long)__shfl_sync(kFull, inc, 31) * p.Hkv;
     }
-    walk_load_seq(p, w);
-    const long long off = lo - before;
-    w.h = (int)(off / w.nt);
-    w.t = (int)(off % w.nt);
-    return true;
+    return lo < hi;
 }
 
 template <int D>
@@ -406,10 +538,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int b = 0; b < p.B; ++b)
             if (p.prefix_len[b] != clamp_prefix(p, b) || p.block_len[b] != clamp_block(p, b))
                 atomicOr(p.status, kStatusClamped);
-    long long N, lo, hi;
+    long long lo, hi;
     Walk w0 = {0, 0, 0, 1, 0, 0};
     // an empty range (only when N < C) runs no loop below
-    const long long ntiles = plan(p, N, lo, hi, w0) ? hi - lo : 0;
+    const long long ntiles = plan(p, lo, hi, w0) ? hi - lo : 0;
 
     if (warp == kProducerWarp) {
         // ================================ producer ===============================
@@ -703,38 +835,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool whole = (seg_first == pair_first) && block_tile;
                 const int pair = ws.b * p.Hkv + ws.h;
                 const size_t slot = (size_t)pair + blockIdx.x;
-                const bool write = owner && row < rows_active;
+                const bool write = row < rows_active;
                 // the row's sum: this thread's half plus its partner's
                 const float l_row = l_sum + __shfl_xor_sync(kFull, l_sum, 16);
                 const float inv = l_row > 0.f ? 1.f / l_row : 0.f;
                 const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;
                 const int gq = row % p.G;
-                uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
-                                          (size_t)ws.h * p.G + gq) * D;
-                float *prow = p.part_o + (slot * p.rows_max + row) * D;
-#pragma unroll 1
-                for (int c = 0; c < D; c += 32) {
-                    float v[32];
-                    tmem_ld32(tmem + lane_base + (uint32_t)(2 * kTileKeys + c), v);
-                    if (write) {
+                // this thread's columns: [64 g + 32 half, +32) for each 64-column group g
+                float v[D / 2];
+                tmem_ld_orow<D>(tmem + lane_base + (uint32_t)(2 * kTileKeys), v);
+                if (write) {
+                    uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
+                                              (size_t)ws.h * p.G + gq) * D + 32 * half;
+                    float *prow = p.part_o + (slot * p.rows_max + row) * D + 32 * half;
+#pragma unroll
+                    for (int g = 0; g < D / 64; ++g) {
+                        const float *x = v + 32 * g;
                         if (whole) {
 #pragma unroll
                             for (int j = 0; j < 32; j += 8)
-                                *reinterpret_cast<uint4 *>(orow + c + j) =
-                                    make_uint4(pack_bf16(v[j] * inv, v[j + 1] * inv),
-                                               pack_bf16(v[j + 2] * inv, v[j + 3] * inv),
-                                               pack_bf16(v[j + 4] * inv, v[j + 5] * inv),
-                                               pack_bf16(v[j + 6] * inv, v[j + 7] * inv));
+                                *reinterpret_cast<uint4 *>(orow + 64 * g + j) =
+                                    make_uint4(pack_bf16(x[j] * inv, x[j + 1] * inv),
+                                               pack_bf16(x[j + 2] * inv, x[j + 3] * inv),
+                                               pack_bf16(x[j + 4] * inv, x[j + 5] * inv),
+                                               pack_bf16(x[j + 6] * inv, x[j + 7] * inv));
                         } else {
 #pragma unroll
                             for (int j = 0; j < 32; j += 4)
-                                *reinterpret_cast<float4 *>(prow + c + j) =
-                                    make_float4(v[j] * inv, v[j + 1] * inv, v[j + 2] * inv,
-                                                v[j + 3] * inv);
+                                *reinterpret_cast<float4 *>(prow + 64 * g + j) =
+                                    make_float4(x[j] * inv, x[j + 1] * inv, x[j + 2] * inv,
+                                                x[j + 3] * inv);
                         }
                     }
                 }
-                if (write) {
+                if (write && owner) {
                     if (whole)
                         p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gq) * p.max_block +
                               irow] = lse;
@@ -793,24 +927,23 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
     const int row = (blockIdx.x % rblocks) * kMergeWarps + warp;
     const int b = pair / p.Hkv, h = pair % p.Hkv;
     const int C = p.num_ctas;
-    long long N = 0, before = 0;
+    // one pass: all tiles, and the tiles of the sequences before b
+    long long total = 0, before = 0;
     for (int b0 = 0; b0 < p.B; b0 += 32) {
-        const int bb = b0 + lane;
-        const long long v = bb < p.B ? (long long)tiles_of(clamp_prefix(p, bb)) * p.Hkv : 0;
-        N += v;
-        if (bb < b) before += v;
+        const int nt = seq_tiles(p, b0 + lane);
+        total += (long long)__reduce_add_sync(kFull, (unsigned)nt) * p.Hkv;
+        before += (long long)__reduce_add_sync(kFull, b0 + lane < b ? (unsigned)nt : 0u) * p.Hkv;
     }
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) {
-        N += __shfl_xor_sync(kFull, N, d);
-        before += __shfl_xor_sync(kFull, before, d);
-    }
+    const Split sp = split_from_total(p, total);
     const int nt = tiles_of(clamp_prefix(p, b));
-    const long long first = before + (long long)h * nt;
-    const int c0 = cta_of(first, N, C);
-    // every nonempty CTA holds a tile when N >= C, so the pair's segments are
-    // those of CTAs c0 .. c1; otherwise each tile is a CTA of its own
-    const int nseg = N >= C ? cta_of(first + nt - 1, N, C) - c0 + 1 : nt;
+    const long long first = before + (long long)h * nt;  // the pair's first tile
+    const long long first_w = first + (long long)sp.beta * pair;
+    const int c0 = cta_of_w(first_w, sp, C);
+    // every CTA holds a tile when beta > 0 or N >= C, so the pair's segments
+    // are those of CTAs c0 .. c1; otherwise (beta = 0) each tile is a CTA of
+    // its own
+    const bool contiguous = sp.beta > 0 || sp.N >= C;
+    const int nseg = contiguous ? cta_of_w(first_w + nt - 1, sp, C) - c0 + 1 : nt;
     const int rows_active = p.G * clamp_block(p, b);
 
     // partials come from the attention grid
@@ -840,7 +973,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
 #pragma unroll
             for (int v = 0; v < VPL; ++v) os[u][v] = 0.f;
             if (s0 + u < nseg) {
-                const int c = N >= C ? c0 + s0 + u : cta_of(first + s0 + u, N, C);
+                const int c = contiguous ? c0 + s0 + u : cta_of_w(first + s0 + u, sp, C);
                 const size_t rs = ((size_t)pair + c) * p.rows_max + row;
                 ls[u] = __ldcg(p.part_lse + rs);
                 const float *src = p.part_o + rs * D + VPL * lane;
@@ -889,15 +1022,15 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
                      const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
                      cudaStream_t stream) {
     constexpr int smem = Layout<D>::kBytes;
-    static bool configured[64] = {false};
+    static std::atomic<bool> configured[64];  // the smem opt-in, once per device
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev < 64 && !configured[dev]) {
+    if (dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
         e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  smem);
         if (e != cudaSuccess) return e;
-        configured[dev] = true;
+        if (dev < 64) configured[dev].store(true, std::memory_order_release);
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)p.num_ctas);
@@ -921,9 +1054,15 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
 }  // namespace tc
 
 int attn_grid_size(int device) {
+    static std::atomic<int> sms_of[64];  // the SM count, looked up once per device
+    if (device >= 0 && device < 64) {
+        const int known = sms_of[device].load(std::memory_order_relaxed);
+        if (known > 0) return known;
+    }
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess)
         return 0;
+    if (device >= 0 && device < 64) sms_of[device].store(sms, std::memory_order_relaxed);
     return sms;
 }
 

@@ -24,6 +24,7 @@ constexpr int kAcceptCtas = 8;
 constexpr int kAcceptThreads = 1024;
 constexpr int kAcceptWarps = kAcceptThreads / 32;
 constexpr int kMaxW = 1024;
+constexpr int kBatch = 8;  // vector loads in flight per thread
 
 // (value, index) order of the argmax: larger value wins, equal values go to
 // the smaller index, so the result is the first maximum.
@@ -78,40 +79,32 @@ __global__ void __launch_bounds__(kAcceptThreads)
         int bi = 0x7fffffff;
         if (i < W) {
             const float *row = logits + ((size_t)b * W + i) * (size_t)vocab + lo;
-            if (VEC == 4) {
-                const float4 *x4 = reinterpret_cast<const float4 *>(row);
-                int j = part;
-                for (; j + 3 * tpr < nvec; j += 4 * tpr) {
-                    float4 a[4];
+            // batches of kBatch vector loads, all issued before the compares
+            for (int j0 = part; j0 < nvec; j0 += kBatch * tpr) {
+                float a[kBatch][VEC];
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) a[u] = __ldcs(x4 + j + u * tpr);
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int e = lo + 4 * (j + u * tpr);
-                        better(bv, bi, a[u].x, e);
-                        better(bv, bi, a[u].y, e + 1);
-                        better(bv, bi, a[u].z, e + 2);
-                        better(bv, bi, a[u].w, e + 3);
+                for (int u = 0; u < kBatch; ++u) {
+                    const int j = j0 + u * tpr;
+                    if (j < nvec) {
+                        if (VEC == 4) {
+                            const float4 x = __ldcs(reinterpret_cast<const float4 *>(row) + j);
+                            a[u][0] = x.x;
+                            a[u][1 % VEC] = x.y;
+                            a[u][2 % VEC] = x.z;
+                            a[u][VEC - 1] = x.w;
+                        } else {
+                            a[u][0] = __ldcs(row + j);
+                        }
                     }
                 }
-                for (; j < nvec; j += tpr) {
-                    const float4 a = __ldcs(x4 + j);
-                    const int e = lo + 4 * j;
-                    better(bv, bi, a.x, e);
-                    better(bv, bi, a.y, e + 1);
-                    better(bv, bi, a.z, e + 2);
-                    better(bv, bi, a.w, e + 3);
-                }
-            } else {
-                int j = part;
-                for (; j + 3 * tpr < nvec; j += 4 * tpr) {
-                    float a[4];
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) a[u] = __ldcs(row + j + u * tpr);
+                for (int u = 0; u < kBatch; ++u) {
+                    const int j = j0 + u * tpr;
+                    if (j < nvec) {
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) better(bv, bi, a[u], lo + j + u * tpr);
+                        for (int e = 0; e < VEC; ++e) better(bv, bi, a[u][e], lo + VEC * j + e);
+                    }
                 }
-                for (; j < nvec; j += tpr) better(bv, bi, __ldcs(row + j), lo + j);
             }
         }
         warp_best(bv, bi);

@@ -54,6 +54,13 @@ def test_split_across_many_ctas():
     run_small(small(batch=2, kv_heads=2, q_heads=8, prefix=(5000, 5000), block=(8,)))
 
 
+@pytest.mark.parametrize("P", [3456, 3457, 9000])
+def test_weighted_split_threshold(P):
+    """8 pairs: the split weights block tiles once the list holds at least
+    (2 + 1) tiles per CTA (P >= 3457 here); both sides of the threshold."""
+    run_small(small(batch=1, kv_heads=8, q_heads=8, prefix=(P, P), block=(8,)))
+
+
 def test_sharp_softmax_scale():
     """scale = 1 makes the softmax peaked (the default 1/sqrt(D) is nearly flat here)."""
     run_small(small(q_heads=8, kv_heads=2, prefix=(500, 500), block=(8,)), scale=1.0)
@@ -156,6 +163,30 @@ def test_workspace_reused_by_back_to_back_calls():
         assert_close(out.float().cpu().numpy(), ref_o, lse.cpu().numpy(), ref_l,
                      where=f"[layer {layer} prefix {pl} block {bl}]")
     assert das.workspace_status(ws) == 0
+
+
+def test_attention_call_object_matches_functional_api():
+    """AttentionCall (arguments checked once) gives the functional calls' bits."""
+    import paper_2609_34538_gb300 as das
+    wl = small(batch=2, q_heads=8, kv_heads=2, prefix=(700, 700), block=(8,))
+    K, V = wl_mod.gen_cache(wl, depths=[2, 8])
+    cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+    ws = das.new_workspace(cache, 8, 8)
+    q = dev_bf16(wl_mod.gen_q(wl, 1))
+    kb, vb = map(dev_bf16, wl_mod.gen_block_kv(wl, 1))
+    pl, bl = dev_i32([700, 650]), dev_i32([8, 3])
+    call = das.AttentionCall(cache, pl, bl, q, kb, vb, ws)
+    o1, l1 = das.das_mature_v_attention(cache, 1, 2, 8, pl, bl, q, kb, vb, ws)
+    o2, l2 = call.mature_v(1, 2, 8)
+    o1, l1, o2, l2 = o1.clone(), l1.clone(), o2.clone(), l2.clone()
+    o3, l3 = das.das_verify_attention(cache, 1, 8, pl, bl, q, kb, vb, ws)
+    o3, l3 = o3.clone(), l3.clone()
+    o4, l4 = call.verify(1, 8)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    assert torch.equal(o3, o4) and torch.equal(l3, l4)
+    with pytest.raises(TypeError):
+        das.AttentionCall(cache, pl, bl, q.float(), kb, vb, ws)
 
 
 def test_host_errors_raise():
