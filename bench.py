@@ -279,9 +279,12 @@ def gpu_arm(args):
     elif e2e is not None:
         e2e.pop("_seconds")
 
-    probes = None
+    probes = seq = None
     if not args.no_probes:
         probes = {n: draft_probe(n, dev, 200, 5, peak) for n in ("long", "batched")}
+        with torch.cuda.stream(stream):
+            pl.copy_(P0)  # the timed steps committed onto the prefix
+        seq = sequential_probe(wl, cache, pl, ws, dev, 20, 3, peak)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -322,6 +325,7 @@ def gpu_arm(args):
                      "kernel": "attn_kernel + merge_kernel (one Mature-V layer call)",
                      "peak_source": f"{peak_kind} HBM copy bandwidth"},
         "long_prefix_draft": probes,
+        "sequential_draft": seq,
         "gpu_launches": K_steps * (2 * L * 2 + 1 + 2),
         "e2e": e2e,
         "cpu_baseline": cpu,
@@ -391,6 +395,71 @@ def draft_probe(name, dev, steps, warmup, peak):
             "per_call_us": round(statistics.mean(ms) * 1e3 / L, 2), "gbs": round(gbs, 1),
             "pct_of_measured_hbm": round(100 * gbs / peak, 1),
             "pct_of_nominal_8000": round(100 * gbs / 8000.0, 1), "steps": len(ms)}
+
+
+def sequential_probe(wl, cache, pl, ws, dev, steps, warmup, peak):
+    """The sequential drafting loop (Sec. 3.2, Eq. 4; App. A.2) on the main
+    workload's cache: a block of T = max_block tokens drafted one at a time;
+    token i runs d = key_depth recurrence steps x L layer calls with block
+    length i, prefix values at depth R and prefix keys at depth s for step s
+    (Mature-V) or at depth R (Deep K/V, Mature-Spec).  The T*d*L calls of one
+    block are one CUDA graph; L2 is flushed before every replay."""
+    import torch
+
+    import paper_2609_34538_gb300 as das
+    from synth import device as sdev
+
+    L, B, T, R, d = wl.layers, wl.batch, wl.max_block, wl.depths, wl.key_depth
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        ins = [sdev.layer_inputs(wl, l, dev) for l in range(L)]
+        outs = [(torch.empty_like(q), torch.empty((B, wl.q_heads, T), dtype=torch.float32,
+                                                  device=dev)) for q, _, _ in ins]
+        bls = [torch.full((B,), i, dtype=torch.int32, device=dev) for i in range(1, T + 1)]
+        flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+    stream.synchronize()
+    res = {}
+    for policy in ("mature_v", "deep_kv"):
+        calls = []
+        for i in range(T):
+            for s in range(1, d + 1):
+                for l in range(L):
+                    q, kb, vb = ins[l]
+                    calls.append(das.AttentionCall(cache, pl, bls[i], q, kb, vb, ws,
+                                                   out=outs[l][0], lse=outs[l][1]))
+        kap = [s for i in range(T) for s in range(1, d + 1) for l in range(L)]
+
+        def block():
+            for c, k, l in zip(calls, kap, [l for _ in range(T * d) for l in range(L)]):
+                c.mature_v(l, k if policy == "mature_v" else R, R, stream=stream)
+
+        with torch.cuda.stream(stream):
+            block()
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            block()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(warmup + steps)]
+        for e0, e1 in ev:
+            with torch.cuda.stream(stream):
+                flush.fill_(1)
+                e0.record(stream)
+                g.replay()
+                e1.record(stream)
+        stream.synchronize()
+        ms = [e0.elapsed_time(e1) for e0, e1 in ev[warmup:]]
+        ncalls = T * d * L
+        nbytes = wl.prefix_bytes_per_layer() * ncalls
+        gbs = nbytes * len(ms) / (sum(ms) / 1e3) / 1e9
+        res[policy] = {"us_per_token": round(statistics.mean(ms) * 1e3 / T, 1),
+                       "us_per_call": round(statistics.mean(ms) * 1e3 / ncalls, 2),
+                       "gbs": round(gbs, 1), "pct_of_measured_hbm": round(100 * gbs / peak, 1)}
+    if das.workspace_status(ws) != 0:
+        raise SystemExit("bench: sequential probe reported a device-side error")
+    del flush
+    return {"calls_per_block": T * d * L, "block_tokens": T, "recurrence_steps": d,
+            "layers": L, **res}
 
 
 def e2e_arm(args, wl, cache, pl, P0, bl, ws, stream, dev):
