@@ -279,12 +279,13 @@ def gpu_arm(args):
     elif e2e is not None:
         e2e.pop("_seconds")
 
-    probes = seq = None
+    probes = seq = wave = None
     if not args.no_probes:
         probes = {n: draft_probe(n, dev, 200, 5, peak) for n in ("long", "batched")}
         with torch.cuda.stream(stream):
             pl.copy_(P0)  # the timed steps committed onto the prefix
         seq = sequential_probe(wl, cache, pl, ws, dev, 20, 3, peak)
+        wave = wave_probe(wl, cache, pl, dev, 20, 3, peak)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -326,6 +327,7 @@ def gpu_arm(args):
                      "peak_source": f"{peak_kind} HBM copy bandwidth"},
         "long_prefix_draft": probes,
         "sequential_draft": seq,
+        "das_wave_refinement": wave,
         "gpu_launches": K_steps * (2 * L * 2 + 1 + 2),
         "e2e": e2e,
         "cpu_baseline": cpu,
@@ -460,6 +462,74 @@ def sequential_probe(wl, cache, pl, ws, dev, steps, warmup, peak):
     del flush
     return {"calls_per_block": T * d * L, "block_tokens": T, "recurrence_steps": d,
             "layers": L, **res}
+
+
+def wave_probe(wl, cache, pl, dev, steps, warmup, peak, gamma=32, w_init=2, rounds=24, k=2,
+               vocab=32000):
+    """DAS-Wave carried parallel refinement (Sec. 3.3) on the main workload's
+    cache with the paper's schedule (gamma 32, W_init 2, J 24; App. A.2) and
+    k recurrent updates per round: J*k*L attention calls with Deep K/V prefix
+    reads over W_j = min(gamma, W_init + j) active rows (Eq. 5), and J shifted
+    readouts over [B][W_j][vocab] logits (Eq. 6).  Synthetic queries, block
+    K/V and logits stand in for the looped model; one CUDA graph per
+    refinement, L2 flushed before every replay."""
+    import torch
+
+    import paper_2609_34538_gb300 as das
+    from synth import device as sdev
+
+    L, B = wl.layers, wl.batch
+    wg = wl.replace(block=(gamma,))
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        ins = [sdev.layer_inputs(wg, l, dev) for l in range(L)]
+        outs = [(torch.empty_like(q), torch.empty((B, wl.q_heads, gamma), dtype=torch.float32,
+                                                  device=dev)) for q, _, _ in ins]
+        lbuf = [torch.randn((B, w, vocab), generator=torch.Generator(device=dev).manual_seed(w),
+                            device=dev, dtype=torch.float32) * 2
+                for w in range(1, gamma + 1)]
+        ws = das.new_workspace(cache, wl.q_heads, gamma, device=dev)
+        anchor = torch.zeros(B, dtype=torch.int32, device=dev)
+        flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+    stream.synchronize()
+    drv = das.WaveRefinement(cache, pl, ws, wl.q_heads, gamma=gamma, w_init=w_init,
+                             rounds=rounds, k_steps=k)
+
+    def step(j, s, layer):
+        q, kb, vb = ins[layer]
+        return q, kb, vb, outs[layer][0], outs[layer][1]
+
+    def refine():
+        drv.run(anchor, step, lambda j: lbuf[drv.widths[j] - 1], stream=stream)
+
+    with torch.cuda.stream(stream):
+        refine()
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        refine()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(warmup + steps)]
+    for e0, e1 in ev:
+        with torch.cuda.stream(stream):
+            flush.fill_(1)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+    stream.synchronize()
+    if das.workspace_status(ws) != 0:
+        raise SystemExit("bench: DAS-Wave probe reported a device-side error")
+    ms = [e0.elapsed_time(e1) for e0, e1 in ev[warmup:]]
+    ncalls = rounds * k * L
+    nbytes = wl.replace(key_depth=wl.depths).prefix_bytes_per_layer() * ncalls
+    gbs = nbytes * len(ms) / (sum(ms) / 1e3) / 1e9
+    del flush, lbuf
+    return {"gamma": gamma, "w_init": w_init, "rounds": rounds, "k": k,
+            "attention_calls": ncalls, "readouts": rounds,
+            "widths": [drv.widths[0], drv.widths[-1]],
+            "us_per_refinement": round(statistics.mean(ms) * 1e3, 1),
+            "us_per_call": round(statistics.mean(ms) * 1e3 / (ncalls + rounds), 2),
+            "attention_gbs": round(gbs, 1), "pct_of_measured_hbm": round(100 * gbs / peak, 1)}
 
 
 def e2e_arm(args, wl, cache, pl, P0, bl, ws, stream, dev):

@@ -158,6 +158,23 @@ das_status das_greedy_accept(const float *logits, const int32_t *draft_ids, int 
                              int32_t *next_token, void *stream);
 
 /*
+ * Shifted token readout of a DAS-Wave refinement round (Sec. 3.3, Eq. 6).
+ * After the k recurrent draft updates of round j over the W = W_j active
+ * positions [x_t, z_1 .. z_{W-1}] (W_j = min(gamma, W_init + j), Eq. 5), the
+ * readout of position i updates the guess of the following position:
+ *   tokens[b][i + 1] = argmax_v logits[b][i][v]   for 0 <= i < W
+ * (smallest index on ties, binary32 comparisons, as das_greedy_accept).
+ * tokens[b][0] (the anchor) and tokens[b][i] for i > W are not written; the
+ * readout of the last active position is the candidate that enters the
+ * window in the next round.
+ *   logits   device fp32 [B][W][vocab]
+ *   tokens   device int32 [B][stride], stride >= W + 1
+ * Requires 1 <= W <= 1024, 1 <= vocab < 2^31.
+ */
+das_status das_wave_readout(const float *logits, int B, int W, int vocab, int32_t *tokens,
+                            int stride, void *stream);
+
+/*
  * Commit (Sec. 3.4; App. B.1): the verifier consumed W inputs
  * [x_t, y_1 .. y_{W-1}] and produced their K/V at every depth and layer.
  * With accepted[b] = a proposals accepted, the first n = min(a + 1, W) inputs

@@ -37,6 +37,8 @@ def lib():
         L.das_oracle_greedy_accept.restype = None
         L.das_oracle_kv_append.argtypes = [p, p, i, i, i, i, i, i, p, p, p, i, p, p]
         L.das_oracle_kv_append.restype = None
+        L.das_oracle_wave_readout.argtypes = [p, i, i, i, p, i]
+        L.das_oracle_wave_readout.restype = None
         _lib = L
     return _lib
 
@@ -105,6 +107,24 @@ def greedy_accept(logits, draft):
     lib().das_oracle_greedy_accept(lg.ctypes.data, dr.ctypes.data, B, W, Vv, acc.ctypes.data,
                                    tid.ctypes.data, nxt.ctypes.data)
     return acc, tid, nxt
+
+
+def wave_readout(logits, tokens):
+    """Eq. 6 shifted readout: tokens' = tokens with tokens'[b][i+1] =
+    argmax logits[b][i] for i < W (first maximum).  logits float32 [B][W][V],
+    tokens int32 [B][S], S >= W + 1; the input is not modified."""
+    lg = np.ascontiguousarray(logits, dtype=np.float32)
+    tk = np.array(tokens, dtype=np.int32, copy=True, order="C")
+    B, W, Vv = lg.shape
+    if tk.shape[0] != B or tk.shape[1] < W + 1:
+        raise ValueError("oracle: tokens must be [B][>= W+1]")
+    lib().das_oracle_wave_readout(lg.ctypes.data, B, W, Vv, tk.ctypes.data, tk.shape[1])
+    return tk
+
+
+def wave_width(gamma, w_init, j):
+    """Active width of refinement round j (Eq. 5): W_j = min(gamma, W_init + j)."""
+    return min(gamma, w_init + j)
 
 
 def kv_append(K, V, k_new, v_new, accepted, prefix_len):

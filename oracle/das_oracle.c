@@ -23,6 +23,8 @@
  *                           kappa = nu = R it is the full-depth verify
  *                           attention of Sec. 3.4 (Eq. 7).
  *   das_oracle_greedy_accept greedy acceptance of Sec. 3.4.
+ *   das_oracle_wave_readout  the shifted token readout of a DAS-Wave
+ *                           refinement round, Eq. 6 (Sec. 3.3).
  *   das_oracle_kv_append     the commit of Sec. 3.4 / App. B.1: keep the K/V of
  *                           accepted, materialized verifier inputs at every
  *                           depth and layer.
@@ -259,6 +261,27 @@ void das_oracle_greedy_accept(const float *logits, const int32_t *draft, int B, 
         accepted[b] = a;
         next_token[b] = a < W ? target_ids[b * W + a] : draft[b * W + W - 1];
     }
+}
+
+/* ---------------------------------------------------------------------------
+ * Shifted readout of a DAS-Wave refinement round (Sec. 3.3, Eq. 6).  After the
+ * k recurrent draft updates of round j over the W_j active positions
+ * [x_t, z_1 .. z_{W_j - 1}], the readout of position i updates the guess of
+ * the following position: z_{i+1} = argmax_v logits[b][i][v] for 0 <= i < W.
+ * tokens is [B][stride] with stride >= W + 1; position 0 (the anchor) and
+ * positions past W are left as they are.  First maximum on ties, binary32
+ * comparisons, as in greedy acceptance.
+ * ------------------------------------------------------------------------- */
+void das_oracle_wave_readout(const float *logits, int B, int W, int vocab, int32_t *tokens,
+                             int stride) {
+    for (int b = 0; b < B; ++b)
+        for (int i = 0; i < W; ++i) {
+            const float *row = logits + ((size_t)b * W + i) * vocab;
+            int best = 0;
+            for (int v = 1; v < vocab; ++v)
+                if (row[v] > row[best]) best = v;
+            tokens[(size_t)b * stride + i + 1] = best;
+        }
 }
 
 /* ---------------------------------------------------------------------------

@@ -11,8 +11,12 @@ ABI in include/das.h:
     das_verify_attention    full-depth verify attention (Sec. 3.4, Eq. 7)
     das_greedy_accept       greedy acceptance (Sec. 3.4)
     das_kv_append           commit of accepted K/V at every depth (App. B.1)
+    das_wave_readout        DAS-Wave shifted token readout (Eq. 6)
     AttentionCall           the attention calls with arguments checked once, for
                             loops that call with the same tensors every step
+    wave_widths, WaveRefinement
+                            DAS-Wave's round schedule (Eq. 5) and the device
+                            side of its carried parallel refinement (Sec. 3.3)
 
 If libdas.so is missing the import fails: there is no fallback.
 """
@@ -56,6 +60,8 @@ def _load():
     lib.das_greedy_accept.restype = i
     lib.das_kv_append.argtypes = [cp, p, p, p, i, p, p, p]
     lib.das_kv_append.restype = i
+    lib.das_wave_readout.argtypes = [p, i, i, i, p, i, p]
+    lib.das_wave_readout.restype = i
     lib.das_mature_v_attention_noalloc.argtypes = [cp, i, i, i, p, p, i, p, p, p, i, f, p, p, p]
     lib.das_mature_v_attention_noalloc.restype = i
     lib.das_status_string.argtypes = [i]
@@ -287,3 +293,72 @@ def das_kv_append(cache, k_new, v_new, accepted, prefix_len, error_flag, stream=
     _check(LIB.das_kv_append(ctypes.byref(cache.desc), _ptr(k_new), _ptr(v_new), _ptr(accepted),
                              W, _ptr(prefix_len), _ptr(error_flag), _stream(stream)),
            "das_kv_append")
+
+
+def das_wave_readout(logits, tokens, stream=None):
+    """Shifted readout of a DAS-Wave round (Eq. 6), in place:
+    tokens[b][i + 1] = argmax_v logits[b][i][v] for i < W; returns tokens."""
+    _need(logits, torch.float32, "logits", 3)
+    _need(tokens, torch.int32, "tokens", 2)
+    B, W, V = logits.shape
+    if tokens.shape[0] != B or tokens.shape[1] < W + 1:
+        raise ValueError("tokens must be [B][>= W + 1] for logits [B][W][vocab]")
+    _check(LIB.das_wave_readout(_ptr(logits), B, W, V, _ptr(tokens), tokens.shape[1],
+                                _stream(stream)), "das_wave_readout")
+    return tokens
+
+
+def wave_widths(gamma, w_init, rounds):
+    """Active widths W_j = min(gamma, W_init + j) of rounds j = 0 .. J-1 (Eq. 5)."""
+    if gamma < 1 or w_init < 1 or w_init > gamma or rounds < 0:
+        raise ValueError("need 1 <= W_init <= gamma and J >= 0")
+    return [min(gamma, w_init + j) for j in range(rounds)]
+
+
+class WaveRefinement:
+    """The device side of DAS-Wave's carried parallel refinement (Sec. 3.3).
+
+    Round j works on the W_j = min(gamma, W_init + j) active positions
+    [x_t, z_1 .. z_{W_j - 1}] (Eq. 5): k recurrent draft updates, each running
+    the L core layers, whose attention reads the verified prefix at Deep K/V
+    (key and value depth R) and the active positions' own K/V under the
+    causal mask; then the shifted readout (Eq. 6) revises the token guesses
+    and the last position's readout becomes the candidate that enters the
+    window next round.  Token guesses start as the repeated anchor.
+
+    The looped model between the attention calls is the caller's:
+      step(j, s, layer) -> (q, k_blk, v_blk, out, lse) buffers of the call
+          (q/out [B][gamma][Hq][D], k_blk/v_blk [B][gamma][Hkv][D],
+          lse [B][Hq][gamma]; rows >= W_j are inactive),
+      logits(j) -> fp32 [B][W_j][vocab] readout logits of round j.
+    After run(), tokens[:, :w] is the verifier input [x_t, y_1 .. y_{w-1}] and
+    tokens[:, w] the final readout y_w, w = W_{J-1}.
+    """
+
+    def __init__(self, cache, prefix_len, workspace, num_q_heads, gamma=32, w_init=2, rounds=24,
+                 k_steps=2):
+        R, L, B, cap, H, D = cache.shape
+        self.cache, self.prefix_len, self.workspace = cache, prefix_len, workspace
+        self.num_q_heads, self.gamma, self.k_steps, self.layers = num_q_heads, gamma, k_steps, L
+        self.widths = wave_widths(gamma, w_init, rounds)
+        dev = cache.k.device
+        # block_len of every distinct width, made once
+        self._bl = {w: torch.full((B,), w, dtype=torch.int32, device=dev)
+                    for w in sorted(set(self.widths))}
+        self.tokens = torch.zeros((B, gamma + 1), dtype=torch.int32, device=dev)
+
+    def run(self, anchor, step, logits, stream=None):
+        """anchor: device int32 [B].  Returns the token buffer [B][gamma + 1]."""
+        R = self.cache.shape[0]
+        s_ = torch.cuda.current_stream() if stream is None else stream
+        with torch.cuda.stream(s_):
+            self.tokens.copy_(anchor.view(-1, 1).expand_as(self.tokens))
+        for j, W in enumerate(self.widths):
+            for s in range(self.k_steps):
+                for layer in range(self.layers):
+                    q, kb, vb, out, lse = step(j, s, layer)
+                    das_mature_v_attention(self.cache, layer, R, R, self.prefix_len,
+                                           self._bl[W], q, kb, vb, self.workspace, out=out,
+                                           lse=lse, stream=s_)
+            das_wave_readout(logits(j), self.tokens, stream=s_)
+        return self.tokens

@@ -242,6 +242,17 @@ das_status das_greedy_accept(const float *logits, const int32_t *draft_ids, int 
                : DAS_ERR_CUDA;
 }
 
+das_status das_wave_readout(const float *logits, int B, int W, int vocab, int32_t *tokens,
+                            int stride, void *stream) {
+    if (!logits || !tokens || B < 0 || W < 1 || W > 1024 || vocab < 1 || stride < W + 1 ||
+        (long long)B * W > 0x7fffffffLL)
+        return DAS_ERR_INVALID_ARG;
+    return das::wave_readout_launch(logits, B, W, vocab, tokens, stride,
+                                    static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAS_OK
+               : DAS_ERR_CUDA;
+}
+
 das_status das_kv_append(const das_kv_cache *cache, const void *k_new, const void *v_new,
                          const int32_t *accepted, int W, int32_t *prefix_len,
                          int32_t *error_flag, void *stream) {

@@ -13,13 +13,16 @@ namespace cg = cooperative_groups;
 namespace das {
 namespace {
 
-// ---- greedy acceptance --------------------------------------------------------
+// ---- greedy acceptance and the DAS-Wave readout ------------------------------
 // One cluster of kAcceptCtas CTAs per sequence.  CTA j of the cluster scans
 // slice j of the vocabulary for every row i < W of its sequence and keeps its
 // best (value, index) per row in shared memory; after a cluster barrier CTA 0
 // reads the kAcceptCtas candidates of each row through distributed shared
-// memory, writes target_ids, counts the accepted prefix and writes accepted
-// and next_token.
+// memory and
+//   - accept mode (Sec. 3.4): writes target_ids, counts the accepted prefix
+//     and writes accepted and next_token;
+//   - readout mode (Eq. 6, Sec. 3.3): writes the argmax of row i as the guess
+//     of position i + 1, tokens[b][i + 1].
 constexpr int kAcceptCtas = 8;
 constexpr int kAcceptThreads = 1024;
 constexpr int kAcceptWarps = kAcceptThreads / 32;
@@ -52,12 +55,22 @@ struct AcceptSmem {
     int first_miss;
 };
 
+struct ArgmaxArgs {
+    const float *logits;  // [B][W][vocab]
+    int W, vocab, slice;
+    // accept mode
+    const int32_t *draft;
+    int32_t *accepted, *target_ids, *next_token;
+    // readout mode
+    int32_t *tokens;  // [B][stride]
+    int stride;
+};
+
 // VEC = 4: float4 loads (vocab % 4 == 0 and 16-byte aligned logits), else 1.
-template <int VEC>
-__global__ void __launch_bounds__(kAcceptThreads)
-    accept_kernel(const float *__restrict__ logits, const int32_t *__restrict__ draft, int W,
-                  int vocab, int slice, int32_t *__restrict__ accepted,
-                  int32_t *__restrict__ target_ids, int32_t *__restrict__ next_token) {
+template <int VEC, bool READOUT>
+__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const ArgmaxArgs a) {
+    const float *__restrict__ logits = a.logits;
+    const int W = a.W, vocab = a.vocab, slice = a.slice;
     __shared__ AcceptSmem sm;
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
@@ -139,15 +152,21 @@ __global__ void __launch_bounds__(kAcceptThreads)
             }
             // a row of -inf keeps the sentinel: the first index wins
             const int t = x == 0x7fffffff ? 0 : x;
-            sm.target[i] = t;
-            target_ids[(size_t)b * W + i] = t;
-            if (draft[(size_t)b * W + i] != t) atomicMin(&sm.first_miss, i);
+            if (READOUT) {
+                a.tokens[(size_t)b * a.stride + i + 1] = t;
+            } else {
+                sm.target[i] = t;
+                a.target_ids[(size_t)b * W + i] = t;
+                if (a.draft[(size_t)b * W + i] != t) atomicMin(&sm.first_miss, i);
+            }
         }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            const int a = sm.first_miss;
-            accepted[b] = a;
-            next_token[b] = a < W ? sm.target[a] : draft[(size_t)b * W + W - 1];
+        if (!READOUT) {
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                const int n = sm.first_miss;
+                a.accepted[b] = n;
+                a.next_token[b] = n < W ? sm.target[n] : a.draft[(size_t)b * W + W - 1];
+            }
         }
     }
     cluster.sync();  // CTA 0 has read the others' shared memory
@@ -246,22 +265,47 @@ cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, unsigne
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
 }
 
+cudaError_t argmax_launch(const ArgmaxArgs &a0, int B, bool readout, cudaStream_t stream) {
+    if (B == 0) return cudaSuccess;
+    if (a0.W > kMaxW || B > 0x7fffffff / kAcceptCtas) return cudaErrorInvalidValue;
+    ArgmaxArgs a = a0;
+    const bool vec = (a.vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(a.logits) & 15u) == 0;
+    // slices are whole float4s
+    int slice = (a.vocab + kAcceptCtas - 1) / kAcceptCtas;
+    a.slice = (slice + 3) & ~3;
+    const dim3 grid((unsigned)(B * kAcceptCtas)), block(kAcceptThreads);
+    if (readout)
+        return vec ? launch_pdl(accept_kernel<4, true>, grid, block, kAcceptCtas, stream, a)
+                   : launch_pdl(accept_kernel<1, true>, grid, block, kAcceptCtas, stream, a);
+    return vec ? launch_pdl(accept_kernel<4, false>, grid, block, kAcceptCtas, stream, a)
+               : launch_pdl(accept_kernel<1, false>, grid, block, kAcceptCtas, stream, a);
+}
+
 }  // namespace
 
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream) {
-    if (B == 0) return cudaSuccess;
-    if (W > kMaxW || B > 0x7fffffff / kAcceptCtas) return cudaErrorInvalidValue;
-    const bool vec = (vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(logits) & 15u) == 0;
-    // slices are whole float4s
-    int slice = (vocab + kAcceptCtas - 1) / kAcceptCtas;
-    slice = (slice + 3) & ~3;
-    const dim3 grid((unsigned)(B * kAcceptCtas)), block(kAcceptThreads);
-    return vec ? launch_pdl(accept_kernel<4>, grid, block, kAcceptCtas, stream, logits, draft, W,
-                            vocab, slice, accepted, target_ids, next_token)
-               : launch_pdl(accept_kernel<1>, grid, block, kAcceptCtas, stream, logits, draft, W,
-                            vocab, slice, accepted, target_ids, next_token);
+    ArgmaxArgs a = {};
+    a.logits = logits;
+    a.W = W;
+    a.vocab = vocab;
+    a.draft = draft;
+    a.accepted = accepted;
+    a.target_ids = target_ids;
+    a.next_token = next_token;
+    return argmax_launch(a, B, false, stream);
+}
+
+cudaError_t wave_readout_launch(const float *logits, int B, int W, int vocab, int32_t *tokens,
+                                int stride, cudaStream_t stream) {
+    ArgmaxArgs a = {};
+    a.logits = logits;
+    a.W = W;
+    a.vocab = vocab;
+    a.tokens = tokens;
+    a.stride = stride;
+    return argmax_launch(a, B, true, stream);
 }
 
 cudaError_t append_launch(const das_kv_cache &c, const void *k_new, const void *v_new,

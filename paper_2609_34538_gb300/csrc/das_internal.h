@@ -56,6 +56,10 @@ cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int 
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream);
 
+// tokens[b][i + 1] = argmax of logits[b][i] for i < W (Eq. 6 readout).
+cudaError_t wave_readout_launch(const float *logits, int B, int W, int vocab, int32_t *tokens,
+                                int stride, cudaStream_t stream);
+
 cudaError_t append_launch(const das_kv_cache &c, const void *k_new, const void *v_new,
                           const int32_t *accepted, int W, int32_t *prefix_len,
                           int32_t *error_flag, cudaStream_t stream);

@@ -20,7 +20,7 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for n in ["das_workspace_size", "das_mature_v_attention", "das_verify_attention",
-              "das_greedy_accept", "das_kv_append", "das_status_string"]:
+              "das_greedy_accept", "das_kv_append", "das_wave_readout", "das_status_string"]:
         assert n in names
 
 
@@ -55,3 +55,7 @@ def test_host_argument_checks():
     assert L.das_workspace_size(ctypes.byref(c), 8, 16) == 0        # 8 * 16 rows > 64
     assert L.das_greedy_accept(null, null, 1, 0, 10, null, null, null, null) == das.DAS_ERR_INVALID_ARG
     assert L.das_kv_append(ctypes.byref(c), null, null, null, 1, null, null, null) == das.DAS_ERR_INVALID_ARG
+    assert L.das_wave_readout(null, 1, 4, 10, null, 5, null) == das.DAS_ERR_INVALID_ARG
+    dummy = ctypes.c_void_p(256)  # never dereferenced: the checks fail first
+    assert L.das_wave_readout(dummy, 1, 4, 10, dummy, 4, null) == das.DAS_ERR_INVALID_ARG  # stride < W+1
+    assert L.das_wave_readout(dummy, 1, 0, 10, dummy, 4, null) == das.DAS_ERR_INVALID_ARG  # W = 0

@@ -296,3 +296,53 @@ def test_append_overflow_leaves_sequence_untouched():
     assert list(pl2) == [3, 6]                      # seq 0 overflowed, seq 1 fit
     assert np.array_equal(K2[:, :, 0], K[:, :, 0])  # untouched
     assert np.all(K2[:, :, 1, 5] == 7)
+
+
+# ------------------------------ DAS-Wave readout ------------------------------
+
+def test_wave_widths_eq5():
+    """Eq. 5: W_j = min(gamma, W_init + j).  The paper's setting (gamma = 32,
+    W_init = 2, J = 24; App. A.2) grows from 2 to 25 and never reaches gamma;
+    a small gamma caps the width."""
+    assert [oracle.wave_width(32, 2, j) for j in range(24)] == list(range(2, 26))
+    assert [oracle.wave_width(8, 2, j) for j in range(10)] == [2, 3, 4, 5, 6, 7, 8, 8, 8, 8]
+    assert oracle.wave_width(32, 2, 0) == 2
+
+
+def test_wave_readout_is_shifted_first_maximum():
+    """Eq. 6: the readout of position i becomes the guess of position i + 1
+    (numpy.argmax: first maximum); the anchor (position 0) and positions past
+    W keep their values; an all-tied row and an all -inf row read out 0."""
+    rng = np.random.default_rng(11)
+    B, W, Vv, S = 3, 6, 97, 10
+    logits = rng.normal(0, 2, (B, W, Vv)).astype(np.float32)
+    logits[1, 2, :] = 0.5
+    logits[2, 4, :] = -np.inf
+    logits[0, 3, [5, 40]] = 50.0  # a planted tie: index 5 wins
+    tokens = rng.integers(0, Vv, (B, S)).astype(np.int32)
+    out = oracle.wave_readout(logits, tokens)
+    exp = tokens.copy()
+    exp[:, 1:W + 1] = logits.argmax(axis=2)
+    assert np.array_equal(out, exp)
+    assert out[0, 4] == 5 and out[1, 3] == 0 and out[2, 5] == 0
+    assert np.array_equal(out[:, 0], tokens[:, 0]) and np.array_equal(out[:, W + 1:],
+                                                                    tokens[:, W + 1:])
+
+
+def test_wave_rounds_grow_the_window_with_the_last_readout():
+    """Over rounds with W_j from Eq. 5, the candidate that enters the active
+    window at round j + 1 (position W_j) is the readout of the last active
+    position W_j - 1 at round j (Sec. 3.3); earlier guesses are revised in
+    place."""
+    rng = np.random.default_rng(12)
+    gamma, w_init, J, Vv = 6, 2, 7, 50
+    tokens = np.zeros((1, gamma + 1), dtype=np.int32)
+    tokens[0, 0] = 9  # anchor x_t
+    for j in range(J):
+        W = oracle.wave_width(gamma, w_init, j)
+        logits = rng.normal(0, 1, (1, W, Vv)).astype(np.float32)
+        new = oracle.wave_readout(logits, tokens)
+        assert new[0, 0] == 9
+        assert new[0, W] == logits[0, W - 1].argmax()  # next candidate enters at W
+        tokens = new
+    assert oracle.wave_width(gamma, w_init, J - 1) == gamma
