@@ -228,6 +228,57 @@ das_status das_mature_v_attention_noalloc(const das_kv_cache *cache, int layer, 
                                           float softmax_scale, void *out, float *lse,
                                           void *stream);
 
+/*
+ * A depth-indexed cache whose depths below R are stored as 8-bit floats.
+ * The paper has no counterpart: it keeps every depth in the model's precision.
+ * This variant halves the bytes of the shallow-depth stream that Mature-V
+ * reads (keys at depth r < R) while the mature depth R that carries the
+ * values and the verifier's reads at R stays bf16.
+ *   k_top, v_top  device bf16 [layers][batch][capacity][kv_heads][head_dim]:
+ *                 depth R
+ *   k_low, v_low  device e4m3 (OCP FP8 E4M3: 1 sign, 4 exponent bits with
+ *                 bias 7, 3 mantissa bits; no infinities, S.1111.111 is NaN;
+ *                 largest finite 448)
+ *                 [depths - 1][layers][batch][capacity][kv_heads][head_dim]:
+ *                 depth d < R at slab d - 1; may be NULL when depths == 1
+ * All pointers 16-byte aligned; the caller owns the memory.
+ */
+typedef struct {
+    void *k_top;
+    void *v_top;
+    void *k_low;
+    void *v_low;
+    int depths, layers, batch, capacity, kv_heads, head_dim;
+} das_kv_cache_f8;
+
+/* Workspace bytes for das_mature_v_attention_f8 (as das_workspace_size). */
+size_t das_workspace_size_f8(const das_kv_cache_f8 *cache, int num_q_heads, int max_block);
+
+/*
+ * das_mature_v_attention over a das_kv_cache_f8: keys are read at key_depth
+ * and values at value_depth from k_top / v_top (depth R) or from k_low / v_low
+ * (depths below R, e4m3, widened exactly to bf16 before the products), so
+ * Eqs. 2-3 are evaluated on the stored values.  key_depth = value_depth = d
+ * is the verify attention of depth d (Sec. 3.4).  All other arguments,
+ * results and limits as das_mature_v_attention.
+ */
+das_status das_mature_v_attention_f8(const das_kv_cache_f8 *cache, int layer, int key_depth,
+                                     int value_depth, const int32_t *prefix_len,
+                                     const int32_t *block_len, int max_block, const void *q,
+                                     const void *k_blk, const void *v_blk, int num_q_heads,
+                                     float softmax_scale, void *out, float *lse, void *workspace,
+                                     size_t workspace_bytes, void *stream);
+
+/*
+ * das_kv_append into a das_kv_cache_f8: the staged bf16 K/V of depth R are
+ * copied byte for byte; those of depths below R are rounded to e4m3 (round to
+ * nearest, ties to even; magnitudes above 448 saturate to 448; NaN stays NaN).
+ * Arguments and errors as das_kv_append.
+ */
+das_status das_kv_append_f8(const das_kv_cache_f8 *cache, const void *k_new, const void *v_new,
+                            const int32_t *accepted, int W, int32_t *prefix_len,
+                            int32_t *error_flag, void *stream);
+
 /* Static text for a status code. */
 const char *das_status_string(das_status s);
 

@@ -39,6 +39,12 @@ def lib():
         L.das_oracle_kv_append.restype = None
         L.das_oracle_wave_readout.argtypes = [p, i, i, i, p, i]
         L.das_oracle_wave_readout.restype = None
+        L.das_oracle_e4m3_decode_n.argtypes = [p, p, ctypes.c_size_t]
+        L.das_oracle_e4m3_decode_n.restype = None
+        L.das_oracle_e4m3_from_bf16_n.argtypes = [p, p, ctypes.c_size_t]
+        L.das_oracle_e4m3_from_bf16_n.restype = None
+        L.das_oracle_kv_append_f8.argtypes = [p, p, p, p, i, i, i, i, i, i, p, p, p, i, p, p]
+        L.das_oracle_kv_append_f8.restype = None
         _lib = L
     return _lib
 
@@ -107,6 +113,69 @@ def greedy_accept(logits, draft):
     lib().das_oracle_greedy_accept(lg.ctypes.data, dr.ctypes.data, B, W, Vv, acc.ctypes.data,
                                    tid.ctypes.data, nxt.ctypes.data)
     return acc, tid, nxt
+
+
+def e4m3_decode(codes):
+    """e4m3 codes (uint8) -> float64 values, exactly."""
+    c = np.ascontiguousarray(codes, dtype=np.uint8)
+    out = np.empty(c.shape, dtype=np.float64)
+    lib().das_oracle_e4m3_decode_n(c.ctypes.data, out.ctypes.data, c.size)
+    return out
+
+
+def e4m3_from_bf16(bits):
+    """bf16 bits -> e4m3 codes: nearest, ties to even, saturating at +-448."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16)
+    out = np.empty(b.shape, dtype=np.uint8)
+    lib().das_oracle_e4m3_from_bf16_n(b.ctypes.data, out.ctypes.data, b.size)
+    return out
+
+
+def _bf16_bits_exact(x):
+    """float64 values that are exactly bf16 (e4m3 values are) -> bf16 bits."""
+    f = np.ascontiguousarray(x, dtype=np.float32)
+    u = f.view(np.uint32)
+    if np.any((u & 0xFFFF) != 0):
+        raise ValueError("oracle: value is not a bf16 value")
+    return (u >> 16).astype(np.uint16)
+
+
+def widen_f8_cache(top, low):
+    """The depth-indexed bf16 cache [R][L][B][cap][Hkv][D] that an e4m3 cache
+    (top: bf16 bits [L][B][cap][Hkv][D] of depth R; low: e4m3 codes
+    [R-1][L][B][cap][Hkv][D]) stores, every value widened exactly."""
+    top = np.ascontiguousarray(top, dtype=np.uint16)
+    R = 1 + (0 if low is None else low.shape[0])
+    full = np.empty((R,) + top.shape, dtype=np.uint16)
+    full[R - 1] = top
+    if R > 1:
+        full[:R - 1] = _bf16_bits_exact(e4m3_decode(low))
+    return full
+
+
+def attention_f8(k_top, v_top, k_low, v_low, layer, key_depth, value_depth, prefix_len,
+                 block_len, q, k_blk, v_blk, scale=None, nthreads=None):
+    """Eqs. 2-3 on an e4m3 cache: the attention of the values it stores."""
+    return attention(widen_f8_cache(k_top, k_low), widen_f8_cache(v_top, v_low), layer,
+                     key_depth, value_depth, prefix_len, block_len, q, k_blk, v_blk, scale=scale,
+                     nthreads=nthreads)
+
+
+def kv_append_f8(k_top, v_top, k_low, v_low, k_new, v_new, accepted, prefix_len):
+    """The commit into an e4m3 cache; returns new (k_top, v_top, k_low, v_low,
+    prefix_len, error_flag) without touching the inputs."""
+    kt, vt = (np.array(x, dtype=np.uint16, copy=True) for x in (k_top, v_top))
+    kl, vl = (np.array(x, dtype=np.uint8, copy=True) for x in (k_low, v_low))
+    kn, vn = _u16(k_new), _u16(v_new)
+    R, L, B, W, Hkv, D = kn.shape
+    cap = kt.shape[2]
+    acc = np.ascontiguousarray(accepted, dtype=np.int32)
+    pl = np.array(prefix_len, dtype=np.int32, copy=True)
+    flag = np.zeros(1, dtype=np.int32)
+    lib().das_oracle_kv_append_f8(kt.ctypes.data, vt.ctypes.data, kl.ctypes.data, vl.ctypes.data,
+                                  R, L, B, cap, Hkv, D, kn.ctypes.data, vn.ctypes.data,
+                                  acc.ctypes.data, W, pl.ctypes.data, flag.ctypes.data)
+    return kt, vt, kl, vl, pl, int(flag[0])
 
 
 def wave_readout(logits, tokens):

@@ -25,6 +25,12 @@
  *   das_oracle_greedy_accept greedy acceptance of Sec. 3.4.
  *   das_oracle_wave_readout  the shifted token readout of a DAS-Wave
  *                           refinement round, Eq. 6 (Sec. 3.3).
+ *   das_oracle_e4m3_*        the 8-bit storage of depths below R used by the
+ *                           library's e4m3 cache variant (not in the paper):
+ *                           exact decoding, and rounding to nearest-even
+ *                           with saturation at +-448, from the format's
+ *                           definition (OCP FP8 E4M3: bias 7, 3 mantissa
+ *                           bits, no infinities, S.1111.111 = NaN).
  *   das_oracle_kv_append     the commit of Sec. 3.4 / App. B.1: keep the K/V of
  *                           accepted, materialized verifier inputs at every
  *                           depth and layer.
@@ -285,6 +291,55 @@ void das_oracle_wave_readout(const float *logits, int B, int W, int vocab, int32
 }
 
 /* ---------------------------------------------------------------------------
+ * e4m3 (OCP FP8 E4M3): sign s, exponent field e (4 bits, bias 7), mantissa m
+ * (3 bits).  e = 0: (-1)^s m/8 2^-6; otherwise (-1)^s (1 + m/8) 2^(e-7);
+ * e = 15, m = 7 is NaN (no infinities); the largest finite value is 448.
+ * ------------------------------------------------------------------------- */
+double das_oracle_e4m3_decode(uint8_t c) {
+    const int s = c >> 7, e = (c >> 3) & 15, m = c & 7;
+    if (e == 15 && m == 7) return NAN;
+    const double mag = e == 0 ? ldexp((double)m / 8.0, -6) : ldexp(1.0 + m / 8.0, e - 7);
+    return s ? -mag : mag;
+}
+
+/* Nearest e4m3 value, ties to the even mantissa; magnitudes above 448 and
+ * infinities become +-448; NaN becomes 0x7F. */
+uint8_t das_oracle_e4m3_encode(double x) {
+    if (isnan(x)) return 0x7F;
+    const uint8_t s = signbit(x) ? 0x80 : 0x00;
+    const double a = fabs(x);
+    if (a > 448.0) return s | 0x7E;
+    if (a < ldexp(1.0, -6)) {                 /* subnormal range: steps of 2^-9 */
+        const double q = nearbyint(ldexp(a, 9));  /* current mode: to nearest, ties even */
+        return s | (uint8_t)q;                /* q = 8 is the smallest normal, 0x08 */
+    }
+    int E;
+    frexp(a, &E);                             /* a = f 2^E, f in [0.5, 1) */
+    E -= 1;                                   /* a = (1 + t) 2^E, t in [0, 1) */
+    double q = nearbyint(ldexp(a, 3 - E));    /* 8 (1 + t), in [8, 16] */
+    if (q == 16.0) {                          /* rounded up to the next binade */
+        q = 8.0;
+        E += 1;
+    }
+    const int e = E + 7, m = (int)q - 8;
+    if (e > 15 || (e == 15 && m == 7)) return s | 0x7E;
+    return s | (uint8_t)(e << 3) | (uint8_t)m;
+}
+
+void das_oracle_e4m3_decode_n(const uint8_t *in, double *out, size_t n) {
+    for (size_t i = 0; i < n; ++i) out[i] = das_oracle_e4m3_decode(in[i]);
+}
+
+/* bf16 bits -> e4m3 codes (every bf16 value is exact in double). */
+void das_oracle_e4m3_from_bf16_n(const uint16_t *in, uint8_t *out, size_t n) {
+    for (size_t i = 0; i < n; ++i) {
+        union { uint32_t u; float f; } v;
+        v.u = (uint32_t)in[i] << 16;
+        out[i] = das_oracle_e4m3_encode((double)v.f);
+    }
+}
+
+/* ---------------------------------------------------------------------------
  * Commit (Sec. 3.4, App. B.1).  The verifier consumed [x_t, y_1 .. y_{w-1}]
  * and produced their K/V at every depth and core layer, staged as
  * k_new/v_new [depths][layers][batch][w][Hkv][D].  With a_b proposals
@@ -315,6 +370,45 @@ void das_oracle_kv_append(uint16_t *k_cache, uint16_t *v_cache, int depths, int 
                 size_t ss = (((size_t)d * layers + l) * batch + b) * W;
                 memcpy(k_cache + (cs + p) * row, k_new + ss * row, sizeof(uint16_t) * n * row);
                 memcpy(v_cache + (cs + p) * row, v_new + ss * row, sizeof(uint16_t) * n * row);
+            }
+        prefix_len[b] = p + n;
+    }
+}
+
+
+/* ---------------------------------------------------------------------------
+ * The commit into an e4m3 cache (the library's variant, not in the paper):
+ * as das_oracle_kv_append over k_new/v_new [R][L][B][W][Hkv][D] (bf16), with
+ * depth R copied into k_top/v_top [L][B][cap][Hkv][D] (bf16) and depths
+ * d < R rounded (das_oracle_e4m3_encode) into k_low/v_low
+ * [R-1][L][B][cap][Hkv][D] (e4m3).
+ * ------------------------------------------------------------------------- */
+void das_oracle_kv_append_f8(uint16_t *k_top, uint16_t *v_top, uint8_t *k_low, uint8_t *v_low,
+                             int depths, int layers, int batch, int capacity, int Hkv, int D,
+                             const uint16_t *k_new, const uint16_t *v_new, const int32_t *accepted,
+                             int W, int32_t *prefix_len, int32_t *error_flag) {
+    size_t row = (size_t)Hkv * D;
+    for (int b = 0; b < batch; ++b) {
+        int a = accepted[b];
+        if (a < 0) a = 0;
+        int n = a + 1 < W ? a + 1 : W;
+        int p = prefix_len[b];
+        if (p + n > capacity) {
+            *error_flag = 1;
+            continue;
+        }
+        for (int d = 0; d < depths; ++d)
+            for (int l = 0; l < layers; ++l) {
+                size_t ss = (((size_t)d * layers + l) * batch + b) * W;
+                if (d == depths - 1) {
+                    size_t cs = ((size_t)l * batch + b) * capacity;
+                    memcpy(k_top + (cs + p) * row, k_new + ss * row, sizeof(uint16_t) * n * row);
+                    memcpy(v_top + (cs + p) * row, v_new + ss * row, sizeof(uint16_t) * n * row);
+                } else {
+                    size_t cs = (((size_t)d * layers + l) * batch + b) * capacity;
+                    das_oracle_e4m3_from_bf16_n(k_new + ss * row, k_low + (cs + p) * row, n * row);
+                    das_oracle_e4m3_from_bf16_n(v_new + ss * row, v_low + (cs + p) * row, n * row);
+                }
             }
         prefix_len[b] = p + n;
     }

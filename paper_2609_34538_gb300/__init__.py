@@ -12,6 +12,9 @@ ABI in include/das.h:
     das_greedy_accept       greedy acceptance (Sec. 3.4)
     das_kv_append           commit of accepted K/V at every depth (App. B.1)
     das_wave_readout        DAS-Wave shifted token readout (Eq. 6)
+    DepthKVCacheF8, das_mature_v_attention_f8, das_kv_append_f8
+                            the cache variant with depths below R stored as
+                            e4m3 (not in the paper)
     AttentionCall           the attention calls with arguments checked once, for
                             loops that call with the same tensors every step
     wave_widths, WaveRefinement
@@ -43,6 +46,13 @@ class das_kv_cache(ctypes.Structure):
                 ("kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int)]
 
 
+class das_kv_cache_f8(ctypes.Structure):
+    _fields_ = [("k_top", ctypes.c_void_p), ("v_top", ctypes.c_void_p),
+                ("k_low", ctypes.c_void_p), ("v_low", ctypes.c_void_p), ("depths", ctypes.c_int),
+                ("layers", ctypes.c_int), ("batch", ctypes.c_int), ("capacity", ctypes.c_int),
+                ("kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int)]
+
+
 def _load():
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"{LIB_PATH} is not built: run `python -m paper_2609_34538_gb300.build` "
@@ -62,6 +72,13 @@ def _load():
     lib.das_kv_append.restype = i
     lib.das_wave_readout.argtypes = [p, i, i, i, p, i, p]
     lib.das_wave_readout.restype = i
+    cp8 = ctypes.POINTER(das_kv_cache_f8)
+    lib.das_workspace_size_f8.argtypes = [cp8, i, i]
+    lib.das_workspace_size_f8.restype = sz
+    lib.das_mature_v_attention_f8.argtypes = [cp8, i, i, i, p, p, i, p, p, p, i, f, p, p, p, sz, p]
+    lib.das_mature_v_attention_f8.restype = i
+    lib.das_kv_append_f8.argtypes = [cp8, p, p, p, i, p, p, p]
+    lib.das_kv_append_f8.restype = i
     lib.das_mature_v_attention_noalloc.argtypes = [cp, i, i, i, p, p, i, p, p, p, i, f, p, p, p]
     lib.das_mature_v_attention_noalloc.restype = i
     lib.das_status_string.argtypes = [i]
@@ -362,3 +379,78 @@ class WaveRefinement:
                                            lse=lse, stream=s_)
             das_wave_readout(logits(j), self.tokens, stream=s_)
         return self.tokens
+
+
+class DepthKVCacheF8:
+    """A depth-indexed cache with depth R in bf16 (k_top, v_top
+    [layers][batch][capacity][kv_heads][head_dim]) and depths 1..R-1 as e4m3
+    codes (k_low, v_low uint8 [depths-1][layers][batch][capacity][kv_heads][head_dim])."""
+
+    def __init__(self, k_top, v_top, k_low=None, v_low=None):
+        _need(k_top, torch.bfloat16, "k_top", 5)
+        _need(v_top, torch.bfloat16, "v_top", 5)
+        if k_top.shape != v_top.shape:
+            raise ValueError("k_top and v_top shapes differ")
+        L, B, cap, H, D = k_top.shape
+        R = 1
+        if k_low is not None or v_low is not None:
+            _need(k_low, torch.uint8, "k_low", 6)
+            _need(v_low, torch.uint8, "v_low", 6)
+            if k_low.shape != v_low.shape or tuple(k_low.shape[1:]) != tuple(k_top.shape):
+                raise ValueError("k_low / v_low must be [depths-1] + k_top.shape")
+            R = k_low.shape[0] + 1
+        self.k_top, self.v_top, self.k_low, self.v_low = k_top, v_top, k_low, v_low
+        self.desc = das_kv_cache_f8(k_top.data_ptr(), v_top.data_ptr(), _ptr(k_low), _ptr(v_low),
+                                    R, L, B, cap, H, D)
+
+    @classmethod
+    def empty(cls, depths, layers, batch, capacity, kv_heads, head_dim, device="cuda"):
+        top = (layers, batch, capacity, kv_heads, head_dim)
+        low = (depths - 1,) + top
+        mk = lambda shape, dt: torch.empty(shape, dtype=dt, device=device)
+        return cls(mk(top, torch.bfloat16), mk(top, torch.bfloat16),
+                   mk(low, torch.uint8) if depths > 1 else None,
+                   mk(low, torch.uint8) if depths > 1 else None)
+
+    @property
+    def shape(self):
+        d = self.desc
+        return (d.depths, d.layers, d.batch, d.capacity, d.kv_heads, d.head_dim)
+
+
+def new_workspace_f8(cache, num_q_heads, max_block, device=None):
+    n = int(LIB.das_workspace_size_f8(ctypes.byref(cache.desc), num_q_heads, max_block))
+    if n == 0:
+        raise DasError(DAS_ERR_UNSUPPORTED, "das_workspace_size_f8")
+    return torch.zeros(n, dtype=torch.uint8, device=device or cache.k_top.device)
+
+
+def das_mature_v_attention_f8(cache, layer, key_depth, value_depth, prefix_len, block_len, q,
+                              k_blk, v_blk, workspace, out=None, lse=None, softmax_scale=0.0,
+                              stream=None):
+    """das_mature_v_attention on an e4m3 cache (DepthKVCacheF8); returns (out, lse)."""
+    T, Hq, out, lse = _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse,
+                                      workspace)
+    _check(LIB.das_mature_v_attention_f8(
+        ctypes.byref(cache.desc), layer, key_depth, value_depth, _ptr(prefix_len),
+        _ptr(block_len), T, _ptr(q), _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale),
+        _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(stream)),
+        "das_mature_v_attention_f8")
+    return out, lse
+
+
+def das_kv_append_f8(cache, k_new, v_new, accepted, prefix_len, error_flag, stream=None):
+    """The commit into an e4m3 cache: depth R copied, depths below R rounded to
+    e4m3 (nearest, ties to even, saturating at +-448)."""
+    _need(k_new, torch.bfloat16, "k_new", 6)
+    _need(v_new, torch.bfloat16, "v_new", 6)
+    _need(accepted, torch.int32, "accepted", 1)
+    _need(prefix_len, torch.int32, "prefix_len", 1)
+    _need(error_flag, torch.int32, "error_flag")
+    R, L, B, cap, H, D = cache.shape
+    W = k_new.shape[3]
+    if tuple(k_new.shape) != (R, L, B, W, H, D) or k_new.shape != v_new.shape:
+        raise ValueError("k_new / v_new must be [depths][layers][batch][W][kv_heads][head_dim]")
+    _check(LIB.das_kv_append_f8(ctypes.byref(cache.desc), _ptr(k_new), _ptr(v_new),
+                                _ptr(accepted), W, _ptr(prefix_len), _ptr(error_flag),
+                                _stream(stream)), "das_kv_append_f8")

@@ -49,11 +49,11 @@ namespace {
 constexpr uint32_t kFull = 0xffffffffu;
 constexpr unsigned long long kWaitNs = 2000000000ull;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr int kStages = 4;
 constexpr int kSoftWarps = 4;
 constexpr int kProducerWarp = kSoftWarps;     // TMA loads
 constexpr int kMmaWarp = kSoftWarps + 1;      // tcgen05 MMAs
-constexpr int kThreads = (kSoftWarps + 2) * 32;
+constexpr int kConvWarp0 = kSoftWarps + 2;    // e4m3 -> bf16 widening (e4m3 variants)
+constexpr int kConvWarps = 4;
 constexpr int kRows = 64;            // M of every MMA (query rows per pair)
 constexpr int kTmemCols = 256;       // S buffers [0, 128), O [128, 128 + D)
 constexpr float kRescaleLog2 = 8.f;  // move the reference max only beyond 2^8
@@ -449,22 +449,37 @@ __device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w)
     return lo < hi;
 }
 
-template <int D>
+// Shared memory of one CTA.  Keys and values stored as e4m3 (the depths below
+// R in a das_kv_cache_f8) land in the stage as 8-bit tiles [64 keys][D] and
+// are widened by the conversion warps into a bf16 tile per stage, in the
+// 128-byte-swizzled layout the MMAs read; a pair's block tile is bf16 and is
+// loaded straight into that tile.
+template <int D, bool KF8, bool VF8>
 struct Layout {
+    static constexpr bool kConv = KF8 || VF8;
+    static constexpr int kStages = (KF8 && VF8) ? 3 : 4;
+    static constexpr int kThreads = (kSoftWarps + 2 + (kConv ? kConvWarps : 0)) * 32;
     static constexpr int kPanels = D / 64;
-    static constexpr int kTileBytes = kTileKeys * D * 2;  // K or V of one tile
-    static constexpr int kStageBytes = 2 * kTileBytes;
+    static constexpr int kTileBytes = kTileKeys * D * 2;  // a bf16 K or V tile
+    static constexpr int kTile8Bytes = kTileKeys * D;     // an e4m3 tile
+    static constexpr int kKBytes = KF8 ? kTile8Bytes : kTileBytes;  // K part of a stage
+    static constexpr int kVBytes = VF8 ? kTile8Bytes : kTileBytes;  // V part of a stage
+    static constexpr int kStageBytes = kKBytes + kVBytes;
+    static constexpr int kConvBytes = (KF8 ? kTileBytes : 0) + (VF8 ? kTileBytes : 0);
     static constexpr int kQBytes = kPanels * kRows * 128;  // one query buffer
     static constexpr int kPBytes = kRows * kTileKeys * 2;  // one P buffer
     static constexpr int kStagesOff = 0;
-    static constexpr int kQOff = kStages * kStageBytes;
+    static constexpr int kConvOff = kStages * kStageBytes;  // widened tiles, one set per stage
+    static constexpr int kQOff = kConvOff + kStages * kConvBytes;
     static constexpr int kPOff = kQOff + 2 * kQBytes;
     static constexpr int kBarOff = kPOff + 2 * kPBytes;
     // barriers: full[kStages], empty[kStages], qfull[2], qempty[2], sready[2],
-    // sfree[2], pready[2], pvdone[2], drain
-    static constexpr int kNumBars = 2 * kStages + 13;
+    // sfree[2], pready[2], pvdone[2], drain, kready[kStages]
+    static constexpr int kNumBars = 2 * kStages + 13 + kStages;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
+    static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
+                  "swizzled tiles need 1024-byte alignment");
 };
 
 // K-major 128B-swizzled address of bf16 element (row, col) of a [64][64] panel
@@ -472,14 +487,63 @@ __device__ __forceinline__ uint32_t p_chunk_addr(uint32_t base, int row, int chu
     return base + row * 128 + ((chunk ^ (row & 7)) << 4);
 }
 
+// Two e4m3 values (element 0 in bits 0-7) -> bf16x2 (element 0 in the low
+// half): cvt to f16x2 (exact), each f16 to f32 (exact), and the upper half
+// of each f32 is the bf16 (exact: an e4m3 value has at most 4 significant
+// bits and a 4-bit exponent, well inside bf16).  NaN stays NaN.
+__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint32_t x) {
+    uint32_t h2, r;
+    asm("{\n .reg .b16 t;\n cvt.u16.u32 t, %1;\n cvt.rn.f16x2.e4m3x2 %0, t;\n}"
+        : "=r"(h2)
+        : "r"(x));
+    float lo, hi;
+    asm("{\n .reg .b16 a, b;\n mov.b32 {a, b}, %2;\n cvt.f32.f16 %0, a;\n cvt.f32.f16 %1, b;\n}"
+        : "=f"(lo), "=f"(hi)
+        : "r"(h2));
+    asm("prmt.b32 %0, %1, %2, 0x7632;" : "=r"(r) : "r"(__float_as_uint(lo)), "r"(__float_as_uint(hi)));
+    return r;
+}
+
+// Widen an e4m3 tile [64 keys][D] (row-major, as the 8-bit TMA box lands)
+// into the bf16 tile the MMAs read: D / 64 panels of [64 keys][128 bytes],
+// 16-byte chunk j of key r at (j ^ (r % 8)) * 16 (128-byte swizzle).  The 128
+// conversion threads (ct = 0..127) each take 16-element chunks.
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
+__device__ __forceinline__ void widen_tile(uint32_t src, uint32_t dst, int ct) {
+    constexpr int kChunks = kTileKeys * D / 16;
+#pragma unroll
+    for (int i = 0; i < kChunks / (kConvWarps * 32); ++i) {
+        const int c = ct + i * kConvWarps * 32;
+        const int key = c / (D / 16), d0 = (c % (D / 16)) * 16;
+        uint32_t w0, w1, w2, w3;
+        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
+                     : "r"(src + key * D + d0));
+        const uint32_t row = dst + (d0 / 64) * 8192 + key * 128;
+        const int j = (d0 % 64) / 8;  // the first of two 16-byte bf16 chunks
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                         row + ((j ^ (key & 7)) << 4)),
+                     "r"(e4m3x2_to_bf16x2(w0 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w0 >> 16)),
+                     "r"(e4m3x2_to_bf16x2(w1 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w1 >> 16))
+                     : "memory");
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                         row + (((j + 1) ^ (key & 7)) << 4)),
+                     "r"(e4m3x2_to_bf16x2(w2 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w2 >> 16)),
+                     "r"(e4m3x2_to_bf16x2(w3 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w3 >> 16))
+                     : "memory");
+    }
+}
+
+// KF8 / VF8: prefix keys / values are e4m3 (tm_k / tm_v are 8-bit maps).
+template <int D, bool KF8, bool VF8>
+__global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_kb,
                    const __grid_constant__ CUtensorMap tm_vb,
                    const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
-    using Lt = Layout<D>;
+    using Lt = Layout<D, KF8, VF8>;
+    constexpr int kStages = Lt::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~uintptr_t(1023));
@@ -487,7 +551,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t bars = sbase + Lt::kBarOff;
     const uint32_t b_full = bars, b_empty = bars + 8 * kStages, b_qfull = b_empty + 8 * kStages,
                    b_qempty = b_qfull + 16, b_sready = b_qempty + 16, b_sfree = b_sready + 16,
-                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 16;
+                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 16,
+                   b_kready = b_drain + 8;
+    // where the MMAs read stage s's bf16 K and V: the TMA tile, or the tile
+    // the conversion warps widened from e4m3
+    const uint32_t kconv0 = sbase + Lt::kConvOff, vconv0 = kconv0 + (KF8 ? Lt::kTileBytes : 0);
+    auto k_src = [&](int st) {
+        return KF8 ? kconv0 + st * Lt::kConvBytes : sbase + st * Lt::kStageBytes;
+    };
+    auto v_src = [&](int st) {
+        return VF8 ? vconv0 + st * Lt::kConvBytes : sbase + st * Lt::kStageBytes + Lt::kKBytes;
+    };
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(sm + Lt::kMiscOff);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Lt::kMiscOff + 4);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -510,6 +584,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(b_pvdone, 1);
         mbar_init(b_pvdone + 8, 1);
         mbar_init(b_drain, 1);
+        if (Lt::kConv)
+            for (int s = 0; s < kStages; ++s) mbar_init(b_kready + 8 * s, kConvWarps);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -577,22 +653,33 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (ok && elect_one()) {
                 const uint32_t full = b_full + 8 * s;
                 const uint32_t kdst = sbase + Lt::kStagesOff + s * Lt::kStageBytes;
-                const uint32_t vdst = kdst + Lt::kTileBytes;
-                mbar_arrive_expect_tx(full, Lt::kStageBytes);
+                const uint32_t vdst = kdst + Lt::kKBytes;
                 if (wl.t < wl.nt - 1) {
                     const int tok = wl.t * kTileKeys;
+                    mbar_arrive_expect_tx(full, Lt::kStageBytes);
+                    // an e4m3 tile is one {D, 1, 64} box, a bf16 tile D / 64 swizzled panels
+                    if (KF8) {
+                        tma_5d(kdst, &tm_k, full, 0, wl.h, tok, wl.b, p.key_slab, policy);
+                    } else {
 #pragma unroll
-                    for (int dp = 0; dp < Lt::kPanels; ++dp) {
-                        tma_5d(kdst + dp * 8192, &tm_k, full, dp * 64, wl.h, tok, wl.b,
-                               p.key_slab, policy);
-                        tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
-                               p.value_slab, policy);
+                        for (int dp = 0; dp < Lt::kPanels; ++dp)
+                            tma_5d(kdst + dp * 8192, &tm_k, full, dp * 64, wl.h, tok, wl.b,
+                                   p.key_slab, policy);
                     }
-                } else {
+                    if (VF8) {
+                        tma_5d(vdst, &tm_v, full, 0, wl.h, tok, wl.b, p.value_slab, policy);
+                    } else {
+#pragma unroll
+                        for (int dp = 0; dp < Lt::kPanels; ++dp)
+                            tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
+                                   p.value_slab, policy);
+                    }
+                } else {  // the block's own K / V: bf16, straight to where the MMAs read
+                    mbar_arrive_expect_tx(full, 2 * Lt::kTileBytes);
 #pragma unroll
                     for (int dp = 0; dp < Lt::kPanels; ++dp) {
-                        tma_4d(kdst + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
-                        tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
+                        tma_4d(k_src(s) + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
+                        tma_4d(v_src(s) + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
                     }
                 }
             }
@@ -606,8 +693,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         // descriptors are affine in the address: build each base once and add
         // (byte offset >> 4) for buffers and k-steps
         const uint64_t dq0 = sdesc(sbase + Lt::kQOff, 16, 1024);
-        const uint64_t dk0 = sdesc(sbase + Lt::kStagesOff, 16, 1024);
-        const uint64_t dv0 = sdesc(sbase + Lt::kStagesOff + Lt::kTileBytes, 8192, 1024);
+        const uint64_t dk0 = sdesc(k_src(0), 16, 1024);
+        const uint64_t dv0 = sdesc(v_src(0), 8192, 1024);
+        // byte distance between consecutive stages' K (V) tiles
+        constexpr int kKStride = KF8 ? Lt::kConvBytes : Lt::kStageBytes;
+        constexpr int kVStride = VF8 ? Lt::kConvBytes : Lt::kStageBytes;
         const uint64_t dp0 = sdesc(sbase + Lt::kPOff, 16, 1024);
         Walk wsn = w0;  // walk of the next S
         int qseg = -1, qcur = 0;
@@ -620,7 +710,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 p.status);
             }
             const int s = (int)(kn % kStages);
-            ok = ok && wait(b_full + 8 * s, (uint32_t)((kn / kStages) & 1), abort_flag, p.status);
+            // the stage's tiles in bf16: landed, and widened if stored as e4m3
+            ok = ok && wait((Lt::kConv ? b_kready : b_full) + 8 * s,
+                            (uint32_t)((kn / kStages) & 1), abort_flag, p.status);
             if (kn >= 2)
                 ok = ok && wait(b_sfree + 8 * (int)(kn & 1), (uint32_t)(((kn - 2) >> 1) & 1),
                                 abort_flag, p.status);
@@ -629,7 +721,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 fence_after();
                 if (elect_one()) {
                     const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
-                    const uint64_t b0 = dk0 + (uint64_t)((s * Lt::kStageBytes) >> 4);
+                    const uint64_t b0 = dk0 + (uint64_t)((s * kKStride) >> 4);
                     const uint32_t dS = tmem + (uint32_t)((kn & 1) * kTileKeys);
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
@@ -656,7 +748,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (elect_one()) {
                 const int s = (int)(k % kStages);
                 const uint64_t a0 = dp0 + (uint64_t)(((k & 1) * Lt::kPBytes) >> 4);
-                const uint64_t b0 = dv0 + (uint64_t)((s * Lt::kStageBytes) >> 4);
+                const uint64_t b0 = dv0 + (uint64_t)((s * kVStride) >> 4);
                 const uint32_t dO = tmem + 2 * kTileKeys;
 #pragma unroll
                 for (int kk = 0; kk < kTileKeys / 16; ++kk)
@@ -675,6 +767,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         const unsigned long long t0 = globaltimer();
         while (!mbar_try_wait(b_drain, 0) && globaltimer() - t0 < kWaitNs) {
+        }
+    } else if (Lt::kConv && warp >= kConvWarp0) {
+        // ============================ e4m3 -> bf16 ===============================
+        // Widen every prefix tile's e4m3 K (and V) once it has landed, then
+        // release the stage to the MMA warp (kready); block tiles are bf16
+        // already and are only passed on.
+        const int ct = threadIdx.x - kConvWarp0 * 32;
+        Walk wc = w0;
+        bool ok = true;
+        for (long long j = 0; j < ntiles && ok; ++j) {
+            const int s = (int)(j % kStages);
+            ok = wait(b_full + 8 * s, (uint32_t)((j / kStages) & 1), abort_flag, p.status);
+            if (!ok) break;
+            if (wc.t < wc.nt - 1) {
+                if (KF8) widen_tile<D>(sbase + s * Lt::kStageBytes, k_src(s), ct);
+                if (VF8) widen_tile<D>(sbase + s * Lt::kStageBytes + Lt::kKBytes, v_src(s), ct);
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_kready + 8 * s);
+            walk_next(p, wc);
         }
     } else {
         // ================================ softmax ================================
@@ -810,7 +923,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             l_sum += lt;
             // keys past the end of the tile may hold anything: zero their V rows
             if (nvalid < kTileKeys) {
-                const uint32_t vt = sbase + Lt::kStagesOff + s * Lt::kStageBytes + Lt::kTileBytes;
+                const uint32_t vt = v_src(s);
                 const int nzero = (kTileKeys - nvalid) * 8 * Lt::kPanels;  // 16-byte chunks
                 for (int i = threadIdx.x; i < nzero; i += kSoftWarps * 32) {
                     const int panel = i / ((kTileKeys - nvalid) * 8);
@@ -1017,24 +1130,25 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
     if (lane == 0) *lrow = L > 0.f ? M + __logf(L) : -INFINITY;
 }
 
-template <int D>
+template <int D, bool KF8, bool VF8>
 cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
                      const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
                      cudaStream_t stream) {
-    constexpr int smem = Layout<D>::kBytes;
+    using Lt = Layout<D, KF8, VF8>;
+    constexpr int smem = Lt::kBytes;
     static std::atomic<bool> configured[64];  // the smem opt-in, once per device
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
-        e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 smem);
+        e = cudaFuncSetAttribute(attn_kernel<D, KF8, VF8>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         if (dev < 64) configured[dev].store(true, std::memory_order_release);
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)p.num_ctas);
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3(Lt::kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -1042,7 +1156,7 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, attn_kernel<D>, tk, tv, tkb, tvb, tq, p);
+    e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8>, tk, tv, tkb, tvb, tq, p);
     if (e != cudaSuccess) return e;
     cfg.gridDim = dim3((unsigned)((long long)p.B * p.Hkv *
                                   ((p.rows_max + kMergeWarps - 1) / kMergeWarps)));
@@ -1091,11 +1205,20 @@ void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_ma
     p.part_lse = reinterpret_cast<float *>(ws + off);
 }
 
-cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
-                        const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
-                        const CUtensorMap &tm_vb, const CUtensorMap &tm_q, cudaStream_t stream) {
-    if (head_dim == 128) return tc::launch_d<128>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
-    if (head_dim == 64) return tc::launch_d<64>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+cudaError_t attn_launch(const AttnParams &p, int head_dim, bool keys_e4m3, bool values_e4m3,
+                        const CUtensorMap &tm_k, const CUtensorMap &tm_v,
+                        const CUtensorMap &tm_kb, const CUtensorMap &tm_vb,
+                        const CUtensorMap &tm_q, cudaStream_t stream) {
+#define DAS_LAUNCH(D, K8, V8) tc::launch_d<D, K8, V8>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream)
+    if (head_dim == 128) {
+        if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(128, true, true) : DAS_LAUNCH(128, true, false);
+        return values_e4m3 ? DAS_LAUNCH(128, false, true) : DAS_LAUNCH(128, false, false);
+    }
+    if (head_dim == 64) {
+        if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(64, true, true) : DAS_LAUNCH(64, true, false);
+        return values_e4m3 ? DAS_LAUNCH(64, false, true) : DAS_LAUNCH(64, false, false);
+    }
+#undef DAS_LAUNCH
     return cudaErrorInvalidValue;
 }
 

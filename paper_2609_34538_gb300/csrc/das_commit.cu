@@ -225,6 +225,77 @@ __global__ void __launch_bounds__(kCopyThreads)
     }
 }
 
+// Two bf16 (element 0 in the low half) -> two e4m3 (element 0 in bits 0-7):
+// round to nearest, ties to even; beyond +-448 (and +-inf) saturate to +-448.
+__device__ __forceinline__ uint32_t bf16x2_to_e4m3x2(uint32_t w) {
+    const float lo = __uint_as_float(w << 16), hi = __uint_as_float(w & 0xffff0000u);
+    uint32_t r;
+    asm("{\n .reg .b16 t;\n cvt.rn.satfinite.e4m3x2.f32 t, %1, %2;\n cvt.u32.u16 %0, t;\n}"
+        : "=r"(r)
+        : "f"(hi), "f"(lo));
+    return r;
+}
+
+// das_kv_append_f8: as append_copy_kernel, over the staged [R][L][B][W][Hkv][D]
+// K/V; slabs of depth R are copied to the bf16 top tensors, slabs of lower
+// depths rounded to e4m3 (8 bytes per 16-byte bf16 word) into the low ones.
+__global__ void __launch_bounds__(kCopyThreads)
+    append_f8_kernel(uint4 *__restrict__ k_top, uint4 *__restrict__ v_top,
+                     uint2 *__restrict__ k_low, uint2 *__restrict__ v_low,
+                     const uint4 *__restrict__ kn, const uint4 *__restrict__ vn,
+                     const int32_t *__restrict__ accepted, const int32_t *__restrict__ prefix_len,
+                     int depths, int layers, int batch, int capacity, int W, int row_words,
+                     int chunks) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const size_t slab = blockIdx.x / chunks;
+    const int chunk = blockIdx.x % chunks;
+    const int b = (int)(slab % batch);
+    const int dl = (int)(slab / batch), d = dl / layers, l = dl % layers;
+    const int n = append_count(accepted[b], W);
+    const int p = prefix_len[b];
+    if (p < 0 || p + n > capacity) return;  // reported by append_finalize_kernel
+    const int words = n * row_words;
+    const int w0 = chunk * kCopyChunk + threadIdx.x;
+    if (chunk * kCopyChunk >= words) return;
+    const uint4 *ks = kn + slab * W * row_words;
+    const uint4 *vs = vn + slab * W * row_words;
+    uint4 a[kCopyUnroll], c[kCopyUnroll];
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+        const int w = w0 + u * kCopyThreads;
+        if (w < words) {
+            a[u] = __ldcs(ks + w);
+            c[u] = __ldcs(vs + w);
+        }
+    }
+    if (d == depths - 1) {
+        const size_t o = (((size_t)l * batch + b) * capacity + p) * row_words;
+#pragma unroll
+        for (int u = 0; u < kCopyUnroll; ++u) {
+            const int w = w0 + u * kCopyThreads;
+            if (w < words) {
+                k_top[o + w] = a[u];
+                v_top[o + w] = c[u];
+            }
+        }
+    } else {
+        const size_t o = ((((size_t)d * layers + l) * batch + b) * capacity + p) * row_words;
+        auto q8 = [](uint4 x) {
+            return make_uint2(bf16x2_to_e4m3x2(x.x) | bf16x2_to_e4m3x2(x.y) << 16,
+                              bf16x2_to_e4m3x2(x.z) | bf16x2_to_e4m3x2(x.w) << 16);
+        };
+#pragma unroll
+        for (int u = 0; u < kCopyUnroll; ++u) {
+            const int w = w0 + u * kCopyThreads;
+            if (w < words) {
+                k_low[o + w] = q8(a[u]);
+                v_low[o + w] = q8(c[u]);
+            }
+        }
+    }
+}
+
 // Runs once every copy has read prefix_len: grow it or flag the sequence.
 __global__ void append_finalize_kernel(const int32_t *__restrict__ accepted,
                                        int32_t *__restrict__ prefix_len, int batch, int capacity,
@@ -324,6 +395,27 @@ cudaError_t append_launch(const das_kv_cache &c, const void *k_new, const void *
                                static_cast<const uint4 *>(v_new), accepted,
                                static_cast<const int32_t *>(prefix_len), c.batch, c.capacity, W,
                                row_words, chunks);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(append_finalize_kernel, dim3((unsigned)((c.batch + 127) / 128)), dim3(128),
+                      1, stream, accepted, prefix_len, c.batch, c.capacity, W, error_flag);
+}
+
+cudaError_t append_f8_launch(const das_kv_cache_f8 &c, const void *k_new, const void *v_new,
+                             const int32_t *accepted, int W, int32_t *prefix_len,
+                             int32_t *error_flag, cudaStream_t stream) {
+    const int row_words = c.kv_heads * c.head_dim * 2 / 16;
+    const long long slabs = (long long)c.depths * c.layers * c.batch;
+    const long long words = (long long)W * row_words;
+    if (words > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const int chunks = (int)((words + kCopyChunk - 1) / kCopyChunk);
+    if (slabs * chunks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    cudaError_t e = launch_pdl(
+        append_f8_kernel, dim3((unsigned)(slabs * chunks)), dim3(kCopyThreads), 1, stream,
+        static_cast<uint4 *>(c.k_top), static_cast<uint4 *>(c.v_top),
+        static_cast<uint2 *>(c.k_low), static_cast<uint2 *>(c.v_low),
+        static_cast<const uint4 *>(k_new), static_cast<const uint4 *>(v_new), accepted,
+        static_cast<const int32_t *>(prefix_len), c.depths, c.layers, c.batch, c.capacity, W,
+        row_words, chunks);
     if (e != cudaSuccess) return e;
     return launch_pdl(append_finalize_kernel, dim3((unsigned)((c.batch + 127) / 128)), dim3(128),
                       1, stream, accepted, prefix_len, c.batch, c.capacity, W, error_flag);

@@ -48,9 +48,12 @@ void attn_workspace_layout(void *workspace, int batch, int kv_heads, int rows_ma
 // Launch the tcgen05 attention kernel and its split-K merge on `stream`, each
 // a programmatic dependent of the kernel before it; tm_q maps the queries
 // [B][max_block][Hq][D] with a {64, G, max_block, 1} box.
-cudaError_t attn_launch(const AttnParams &p, int head_dim, const CUtensorMap &tm_k,
-                        const CUtensorMap &tm_v, const CUtensorMap &tm_kb,
-                        const CUtensorMap &tm_vb, const CUtensorMap &tm_q, cudaStream_t stream);
+// keys_e4m3 / values_e4m3: tm_k / tm_v map e4m3 prefix tiles (8-bit maps with
+// a {D, 1, 64, 1, 1} box, no swizzle) instead of bf16 ones.
+cudaError_t attn_launch(const AttnParams &p, int head_dim, bool keys_e4m3, bool values_e4m3,
+                        const CUtensorMap &tm_k, const CUtensorMap &tm_v,
+                        const CUtensorMap &tm_kb, const CUtensorMap &tm_vb,
+                        const CUtensorMap &tm_q, cudaStream_t stream);
 
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
@@ -63,5 +66,11 @@ cudaError_t wave_readout_launch(const float *logits, int B, int W, int vocab, in
 cudaError_t append_launch(const das_kv_cache &c, const void *k_new, const void *v_new,
                           const int32_t *accepted, int W, int32_t *prefix_len,
                           int32_t *error_flag, cudaStream_t stream);
+
+// das_kv_append_f8: depth R copied to the bf16 top tensors, depths below R
+// rounded to e4m3 into the low tensors.
+cudaError_t append_f8_launch(const das_kv_cache_f8 &c, const void *k_new, const void *v_new,
+                             const int32_t *accepted, int W, int32_t *prefix_len,
+                             int32_t *error_flag, cudaStream_t stream);
 
 }  // namespace das

@@ -33,6 +33,8 @@ def host_lib():
         lib.synth_uniform_int.restype = ctypes.c_int64
         lib.synth_accept_inputs.argtypes = [u64, i, i, i, p, p, p]
         lib.synth_accept_inputs.restype = i
+        lib.synth_e4m3_codes.argtypes = [u64, i, u64, ctypes.c_size_t, p]
+        lib.synth_e4m3_codes.restype = None
         _host = lib
     return _host
 
@@ -77,6 +79,18 @@ def normal_block(seed, tensor, layer, b, t0, t1, h0, h1, D, divisor=1.0, nthread
     if rc:
         raise ValueError("coordinates outside the generator's counter layout")
     return out
+
+
+T_KLOW, T_VLOW = 14, 15
+
+
+def e4m3_codes(seed, tensor, shape, c0=0):
+    """uint8 e4m3 codes of the given shape (random sign, exponent field 4..9,
+    random mantissa; never NaN) from tensor stream `tensor`."""
+    n = int(np.prod(shape))
+    out = np.empty(n, dtype=np.uint8)
+    host_lib().synth_e4m3_codes(seed, tensor, c0, n, out.ctypes.data)
+    return out.reshape(shape)
 
 
 def uniform_int(seed, tensor, idx, lo, hi):

@@ -60,7 +60,9 @@ enum {
     SYNTH_T_ACCEPT = 10,
     SYNTH_T_PREFIX = 11,
     SYNTH_T_BLOCK = 12,
-    SYNTH_T_FILL = 13
+    SYNTH_T_FILL = 13,
+    SYNTH_T_KLOW = 14,
+    SYNTH_T_VLOW = 15
 };
 
 SYNTH_FN uint64_t synth_mix(uint64_t z) {

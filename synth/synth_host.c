@@ -145,3 +145,17 @@ void synth_normal_array(uint64_t seed, int tensor, uint64_t c0, size_t n, double
     uint64_t key = synth_key(seed, (uint64_t)tensor);
     for (size_t i = 0; i < n; ++i) out[i] = synth_normal(key, c0 + i);
 }
+
+/*
+ * 8-bit float codes for e4m3 cache contents, drawn (not rounded from
+ * anything): out[i] = sign | exponent field | mantissa from output c0 + i + 1
+ * of tensor stream `tensor`, with the exponent field in 4..9 (magnitudes
+ * 2^-3 .. 1.875 * 2^2), so no code is NaN.
+ */
+void synth_e4m3_codes(uint64_t seed, int tensor, uint64_t c0, size_t n, uint8_t *out) {
+    const uint64_t key = synth_key(seed, (uint64_t)tensor);
+    for (size_t i = 0; i < n; ++i) {
+        const uint64_t r = synth_out(key, c0 + i + 1);
+        out[i] = (uint8_t)(((r >> 63) << 7) | ((4 + (r >> 40) % 6) << 3) | (r & 7));
+    }
+}

@@ -1,0 +1,113 @@
+"""The e4m3 cache variant (depths below R stored as 8-bit floats; not in the
+paper): das_mature_v_attention_f8 against the oracle on the stored values,
+for every combination of e4m3 / bf16 keys and values, and das_kv_append_f8
+bit-exact against the oracle's rounding."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from synth import workloads as wl_mod
+from tests.gpu_util import assert_close, dev_bf16, dev_i32, host_bits
+
+pytestmark = pytest.mark.gpu
+
+
+def small(**kw):
+    base = dict(name="f8", batch=2, layers=2, q_heads=8, kv_heads=2, head_dim=128, depths=6,
+                key_depth=2, value_depth=6, prefix=(700, 700), block=(8,))
+    base.update(kw)
+    return wl_mod.Workload(**base)
+
+
+def host_f8_cache(wl):
+    R = wl.depths
+    K, V = wl_mod.gen_cache(wl, depths=[R])
+    low = (R - 1, wl.layers, wl.batch, wl.capacity, wl.kv_heads, wl.head_dim)
+    return (K[R - 1].copy(), V[R - 1].copy(), synth.e4m3_codes(wl.seed, synth.T_KLOW, low),
+            synth.e4m3_codes(wl.seed, synth.T_VLOW, low))
+
+
+def run_f8(wl, kap, nu, layer=1, prefix=None, block=None, poison_tail=False, scale=0.0):
+    import paper_2609_34538_gb300 as das
+    kt, vt, kl, vl = host_f8_cache(wl)
+    pl = wl.prefix_lens() if prefix is None else np.asarray(prefix, np.int32)
+    bl = wl.block_lens() if block is None else np.asarray(block, np.int32)
+    if poison_tail:  # positions past the prefix hold NaN: never read
+        for b in range(wl.batch):
+            kl[:, :, b, pl[b]:] = 0x7F
+            vl[:, :, b, pl[b]:] = 0x7F
+            kt[:, b, pl[b]:] = 0x7FC0
+            vt[:, b, pl[b]:] = 0x7FC0
+    q = wl_mod.gen_q(wl, layer)
+    kb, vb = wl_mod.gen_block_kv(wl, layer)
+    ref_o, ref_l = oracle.attention_f8(kt, vt, kl, vl, layer, kap, nu, pl, bl, q, kb, vb,
+                                       scale=scale if scale > 0 else None)
+    up8 = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    cache = das.DepthKVCacheF8(dev_bf16(kt), dev_bf16(vt), up8(kl), up8(vl))
+    ws = das.new_workspace_f8(cache, wl.q_heads, wl.max_block)
+    out, lse = das.das_mature_v_attention_f8(cache, layer, kap, nu, dev_i32(pl), dev_i32(bl),
+                                             dev_bf16(q), dev_bf16(kb), dev_bf16(vb), ws,
+                                             softmax_scale=scale)
+    torch.cuda.synchronize()
+    assert_close(out.float().cpu().numpy(), ref_o, lse.cpu().numpy(), ref_l,
+                 where=f"[f8 kappa {kap} nu {nu}]")
+    assert das.workspace_status(ws) == 0
+
+
+@pytest.mark.parametrize("kap,nu", [(2, 6), (3, 3), (6, 2), (6, 6), (1, 5)])
+def test_read_policies_on_e4m3_cache(kap, nu):
+    """Mature-V (e4m3 keys, bf16 values), a low-depth verify (both e4m3),
+    Deep K (bf16 keys, e4m3 values), Deep K/V (both bf16) and another
+    e4m3-key case."""
+    run_f8(small(), kap, nu)
+
+
+@pytest.mark.parametrize("P", [0, 1, 63, 64, 65, 1000])
+def test_prefix_lengths_e4m3(P):
+    run_f8(small(prefix=(P, P)), 2, 6, prefix=[P, max(P - 1, 0)], block=[8, 5])
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_head_dims_e4m3(D):
+    run_f8(small(head_dim=D), 2, 6)
+    run_f8(small(head_dim=D), 3, 3)
+
+
+def test_nan_past_the_prefix_is_never_read_e4m3():
+    run_f8(small(prefix=(300, 300)), 2, 6, prefix=[300, 129], block=[8, 3], poison_tail=True)
+    run_f8(small(prefix=(300, 300)), 4, 4, prefix=[300, 129], block=[8, 3], poison_tail=True)
+
+
+def test_split_across_many_ctas_e4m3():
+    run_f8(small(batch=1, kv_heads=1, q_heads=4, prefix=(20000, 20000), block=(16,)), 2, 6)
+
+
+def test_sharp_scale_e4m3():
+    run_f8(small(), 2, 6, scale=1.0)
+
+
+def test_append_e4m3_bit_exact():
+    import paper_2609_34538_gb300 as das
+    wl = small(batch=3, prefix=(40, 40), block=(8,))
+    R, L, B, W = wl.depths, wl.layers, wl.batch, 6
+    kt, vt, kl, vl = host_f8_cache(wl)
+    kn = np.stack([synth.matured_block(wl.seed + 7, synth.T_KNEW, 0, d, R, l, b, 0, W, 0,
+                                       wl.kv_heads, wl.head_dim)
+                   for d in range(1, R + 1) for l in range(L) for b in range(B)])
+    kn = kn.reshape(R, L, B, W, wl.kv_heads, wl.head_dim)
+    vn = np.ascontiguousarray(kn[::-1])
+    acc = np.array([0, 3, W], np.int32)
+    pl = np.array([40, 10, 5], np.int32)
+    ekt, evt, ekl, evl, epl, eflag = oracle.kv_append_f8(kt, vt, kl, vl, kn, vn, acc, pl)
+    up8 = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    cache = das.DepthKVCacheF8(dev_bf16(kt), dev_bf16(vt), up8(kl), up8(vl))
+    dpl, flag = dev_i32(pl), torch.zeros(1, dtype=torch.int32, device="cuda")
+    das.das_kv_append_f8(cache, dev_bf16(kn), dev_bf16(vn), dev_i32(acc), dpl, flag)
+    torch.cuda.synchronize()
+    assert int(flag.item()) == eflag
+    assert np.array_equal(dpl.cpu().numpy(), epl)
+    assert np.array_equal(host_bits(cache.k_top), ekt) and np.array_equal(host_bits(cache.v_top), evt)
+    assert np.array_equal(cache.k_low.cpu().numpy(), ekl)
+    assert np.array_equal(cache.v_low.cpu().numpy(), evl)

@@ -346,3 +346,90 @@ def test_wave_rounds_grow_the_window_with_the_last_readout():
         assert new[0, W] == logits[0, W - 1].argmax()  # next candidate enters at W
         tokens = new
     assert oracle.wave_width(gamma, w_init, J - 1) == gamma
+
+
+# --------------------------- e4m3 storage (variant) ---------------------------
+
+def _torch_e4m3():
+    torch = pytest.importorskip("torch")
+    if not hasattr(torch, "float8_e4m3fn"):
+        pytest.skip("torch without float8_e4m3fn")
+    return torch
+
+
+def test_e4m3_decode_matches_torch_on_every_code():
+    torch = _torch_e4m3()
+    codes = np.arange(256, dtype=np.uint8)
+    ours = oracle.e4m3_decode(codes)
+    ref = torch.from_numpy(codes).view(torch.float8_e4m3fn).float().double().numpy()
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(ours), nan) and nan.sum() == 2   # S.1111.111 only
+    assert np.array_equal(ours[~nan], ref[~nan])
+    assert ours[0x7E] == 448.0 and ours[0x01] == 2.0 ** -9 and ours[0x08] == 2.0 ** -6
+
+
+def test_e4m3_encode_round_trip_and_torch_rounding():
+    """Every finite code survives decode -> encode; random bf16 values within
+    +-448 round like torch's float -> float8_e4m3fn cast (nearest, ties to
+    even)."""
+    torch = _torch_e4m3()
+    codes = np.array([c for c in range(256) if c not in (0x7F, 0xFF)], dtype=np.uint8)
+    bits = (oracle.e4m3_decode(codes).astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    assert np.array_equal(oracle.e4m3_from_bf16(bits), codes)
+    rng = np.random.default_rng(21)
+    x = np.concatenate([rng.normal(0, s, 20000) for s in (1e-3, 0.1, 1.0, 30.0)])
+    x = np.clip(x, -448, 448).astype(np.float32)
+    b16 = (x.view(np.uint32) >> 16).astype(np.uint16)           # truncate to bf16 values
+    xv = (b16.astype(np.uint32) << 16).view(np.float32)
+    ref = torch.from_numpy(xv).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(oracle.e4m3_from_bf16(b16), ref)
+
+
+def test_e4m3_encode_ties_and_saturation():
+    def enc(v):
+        b = (np.array([v], np.float32).view(np.uint32) >> 16).astype(np.uint16)
+        return int(oracle.e4m3_from_bf16(b)[0])
+    u = 2.0 ** -9                                   # the subnormal step
+    assert [enc(0.5 * u), enc(1.5 * u), enc(2.5 * u), enc(7.5 * u)] == [0x00, 0x02, 0x02, 0x08]
+    assert enc(1.0625) == 0x38 and enc(1.1875) == 0x3A   # ties to the even mantissa
+    assert [enc(448.0), enc(449.0), enc(464.0), enc(1e30), enc(np.inf)] == [0x7E] * 5
+    assert [enc(-449.0), enc(-np.inf)] == [0xFE, 0xFE]
+    assert enc(-0.0) == 0x80
+
+
+def test_e4m3_cache_attention_reduces_to_bf16():
+    """With every depth below R holding e4m3-representable bf16 values, the
+    e4m3 cache is the same cache: attention_f8 equals attention bit for bit;
+    key_depth = value_depth = R reads only the bf16 top."""
+    rng = np.random.default_rng(22)
+    R, L, B, cap, H, D = 3, 1, 2, 40, 2, 8
+    codes = rng.integers(0, 256, (R - 1, L, B, cap, H, D)).astype(np.uint8)
+    codes[(codes & 0x7F) == 0x7F] = 0x38            # no NaN
+    low_bits = (oracle.e4m3_decode(codes).astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    top = rng.integers(0x3C00, 0x4000, (L, B, cap, H, D)).astype(np.uint16)
+    K = np.concatenate([low_bits, top[None]])
+    q = rng.integers(0x3C00, 0x3F80, (B, 4, H, D)).astype(np.uint16)
+    kb = rng.integers(0x3C00, 0x3F80, (B, 4, H, D)).astype(np.uint16)
+    pl, bl = np.array([33, 7], np.int32), np.array([4, 2], np.int32)
+    for kap, nu in [(1, 3), (2, 2), (3, 3), (1, 1)]:
+        o1, l1 = oracle.attention_f8(top, top, codes, codes, 0, kap, nu, pl, bl, q, kb, kb)
+        o2, l2 = oracle.attention(K, K, 0, kap, nu, pl, bl, q, kb, kb)
+        assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
+
+
+def test_e4m3_append_rounds_low_depths_and_copies_the_top():
+    rng = np.random.default_rng(23)
+    R, L, B, cap, H, D, W = 3, 2, 2, 10, 1, 8, 4
+    kt = rng.integers(0, 65535, (L, B, cap, H, D)).astype(np.uint16)
+    kl = rng.integers(0, 255, (R - 1, L, B, cap, H, D)).astype(np.uint8)
+    x = rng.normal(0, 3, (R, L, B, W, H, D)).astype(np.float32)
+    kn = (x.view(np.uint32) >> 16).astype(np.uint16)
+    acc, pl = np.array([1, 5], np.int32), np.array([2, 6], np.int32)
+    kt2, vt2, kl2, vl2, pl2, flag = oracle.kv_append_f8(kt, kt, kl, kl, kn, kn, acc, pl)
+    n = [2, 4]
+    assert flag == 0 and list(pl2) == [4, 10]
+    ekt, ekl = kt.copy(), kl.copy()
+    for b in range(B):
+        ekt[:, b, pl[b]:pl[b] + n[b]] = kn[R - 1, :, b, :n[b]]
+        ekl[:, :, b, pl[b]:pl[b] + n[b]] = oracle.e4m3_from_bf16(kn[:R - 1, :, b, :n[b]])
+    assert np.array_equal(kt2, ekt) and np.array_equal(kl2, ekl)
