@@ -279,13 +279,18 @@ def gpu_arm(args):
     elif e2e is not None:
         e2e.pop("_seconds")
 
-    probes = seq = wave = None
+    probes = seq = wave = f8 = None
     if not args.no_probes:
         probes = {n: draft_probe(n, dev, 200, 5, peak) for n in ("long", "batched")}
         with torch.cuda.stream(stream):
             pl.copy_(P0)  # the timed steps committed onto the prefix
         seq = sequential_probe(wl, cache, pl, ws, dev, 20, 3, peak)
         wave = wave_probe(wl, cache, pl, dev, 20, 3, peak)
+        f8 = {n: f8_probe(n, dev, 200, 5, peak) for n in ("decode", "long")}
+        for n, r in f8.items():
+            bf16_us = (probes[n]["per_call_us"] if n in probes
+                       else statistics.mean(draft_ms) * 1e3 / L)
+            r["speedup_vs_bf16_cache"] = round(bf16_us / r["per_call_us"], 3)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -328,6 +333,7 @@ def gpu_arm(args):
         "long_prefix_draft": probes,
         "sequential_draft": seq,
         "das_wave_refinement": wave,
+        "e4m3_cache_draft": f8,
         "gpu_launches": K_steps * (2 * L * 2 + 1 + 2),
         "e2e": e2e,
         "cpu_baseline": cpu,
@@ -397,6 +403,71 @@ def draft_probe(name, dev, steps, warmup, peak):
             "per_call_us": round(statistics.mean(ms) * 1e3 / L, 2), "gbs": round(gbs, 1),
             "pct_of_measured_hbm": round(100 * gbs / peak, 1),
             "pct_of_nominal_8000": round(100 * gbs / 8000.0, 1), "steps": len(ms)}
+
+
+def f8_probe(name, dev, steps, warmup, peak):
+    """Mature-V draft phase of workload `name` on the e4m3 cache variant
+    (keys at depth r stored as e4m3, values at depth R as bf16; not in the
+    paper), timed like the bf16 probes; bytes per call count 1 byte per key
+    element and 2 per value element."""
+    import torch
+
+    import paper_2609_34538_gb300 as das
+    from synth import device as sdev
+    from synth import workloads as wlm
+
+    wl = wlm.WORKLOADS[name].replace(depths=2, key_depth=1, value_depth=2)
+    L, B, W = wl.layers, wl.batch, wl.max_block
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        cache = das.DepthKVCacheF8.empty(2, L, B, wl.capacity, wl.kv_heads, wl.head_dim,
+                                         device=dev)
+        sdev.fill_matured(cache.v_top, wl.seed, 2, 1, 2, 2)
+        sdev.fill_matured(cache.k_top, wl.seed, 1, 0, 2, 2)
+        g = torch.Generator(device=dev).manual_seed(wl.seed)
+        for t in (cache.k_low, cache.v_low):  # codes with exponent fields 4..9, random sign
+            t.copy_(torch.randint(0x20, 0x50, t.shape, generator=g, device=dev, dtype=torch.int32)
+                    .bitwise_or_(torch.randint(0, 2, t.shape, generator=g, device=dev,
+                                               dtype=torch.int32) * 0x80).to(torch.uint8))
+        pl = torch.from_numpy(wl.prefix_lens()).to(dev)
+        bl = torch.from_numpy(wl.block_lens()).to(dev)
+        ws = das.new_workspace_f8(cache, wl.q_heads, W, device=dev)
+        ins = [sdev.layer_inputs(wl, l, dev) for l in range(L)]
+        outs = [(torch.empty_like(q), torch.empty((B, wl.q_heads, W), dtype=torch.float32,
+                                                  device=dev)) for q, _, _ in ins]
+        flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
+    stream.synchronize()
+
+    def phase():
+        for l, (q, kb, vb) in enumerate(ins):
+            das.das_mature_v_attention_f8(cache, l, 1, 2, pl, bl, q, kb, vb, ws, out=outs[l][0],
+                                          lse=outs[l][1], stream=stream)
+
+    with torch.cuda.stream(stream):
+        phase()
+    stream.synchronize()
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr, stream=stream):
+        phase()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(warmup + steps)]
+    for e0, e1 in ev:
+        with torch.cuda.stream(stream):
+            flush.fill_(1)
+            e0.record(stream)
+            gr.replay()
+            e1.record(stream)
+    stream.synchronize()
+    if das.workspace_status(ws) != 0:
+        raise SystemExit(f"bench: e4m3 {name} probe reported a device-side error")
+    ms = [e0.elapsed_time(e1) for e0, e1 in ev[warmup:]]
+    nbytes = wl.prefix_bytes_per_layer() * 3 // 4 * L  # K 1 byte + V 2 bytes per element pair
+    gbs = nbytes * len(ms) / (sum(ms) / 1e3) / 1e9
+    del cache, flush
+    torch.cuda.empty_cache()
+    return {"workload": wl.name, "storage": "keys e4m3 (depth r), values bf16 (depth R)",
+            "per_call_us": round(statistics.mean(ms) * 1e3 / L, 2), "gbs": round(gbs, 1),
+            "pct_of_measured_hbm": round(100 * gbs / peak, 1), "steps": len(ms)}
 
 
 def sequential_probe(wl, cache, pl, ws, dev, steps, warmup, peak):

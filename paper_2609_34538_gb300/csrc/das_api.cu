@@ -43,10 +43,16 @@ bool encode_uncached(CUtensorMap *m, void *base, int rank, const cuuint64_t *dim
         strides[i] = s;
     }
     cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    // L2 promotion no wider than one contiguous row: the rows of one head are
+    // strided by the other heads, so a 256-byte promotion of a 128-byte row
+    // (an e4m3 row of 128 dims, a bf16 row of 64) fetches a neighbour's row too.
+    const cuuint64_t row_bytes = dims[0] * (e4m3 ? 1 : 2);
+    const CUtensorMapL2promotion promo = row_bytes >= 256   ? CU_TENSOR_MAP_L2_PROMOTION_L2_256B
+                                         : row_bytes >= 128 ? CU_TENSOR_MAP_L2_PROMOTION_L2_128B
+                                                            : CU_TENSOR_MAP_L2_PROMOTION_L2_64B;
     return fn(m, e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
               (cuuint32_t)rank, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-              e4m3 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              e4m3 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B, promo,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 

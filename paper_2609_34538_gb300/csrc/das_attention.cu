@@ -111,6 +111,15 @@ __device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity, volatile int
     return wait_slow(bar, parity, abort_flag, status);
 }
 
+// On the abort path only: wait (at most 20 ms, whatever the abort flag says)
+// for a phase whose completion also means that the copies signalling it
+// have landed, so that no bulk copy into shared memory outlives the CTA.
+__device__ __noinline__ void drain_wait(uint32_t bar, uint32_t parity) {
+    const unsigned long long t0 = globaltimer();
+    while (!mbar_try_wait(bar, parity) && globaltimer() - t0 < 20000000ull) {
+    }
+}
+
 __device__ __forceinline__ void tma_5d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
                                        int c1, int c2, int c3, int c4, uint64_t policy) {
     asm volatile(
@@ -451,13 +460,17 @@ __device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w)
 
 // Shared memory of one CTA.  Keys and values stored as e4m3 (the depths below
 // R in a das_kv_cache_f8) land in the stage as 8-bit tiles [64 keys][D] and
-// are widened by the conversion warps into a bf16 tile per stage, in the
-// 128-byte-swizzled layout the MMAs read; a pair's block tile is bf16 and is
-// loaded straight into that tile.
+// are widened by the conversion warps into bf16 tiles, in the
+// 128-byte-swizzled layout the MMAs read, held in a ring of kConvSlots slots
+// (tile j in slot j % kConvSlots) rather than one per stage: the smaller
+// stages then fit 6 (or 7) deep instead of 4, which is what keeps more DRAM
+// requests in flight per SM.  A pair's block tile is bf16 and is loaded
+// straight into its ring slot (or, for bf16 operands, into the stage).
 template <int D, bool KF8, bool VF8>
 struct Layout {
     static constexpr bool kConv = KF8 || VF8;
-    static constexpr int kStages = (KF8 && VF8) ? 3 : 4;
+    static constexpr int kStages = (KF8 && VF8) ? 7 : kConv ? 6 : 4;
+    static constexpr int kConvSlots = 2;
     static constexpr int kThreads = (kSoftWarps + 2 + (kConv ? kConvWarps : 0)) * 32;
     static constexpr int kPanels = D / 64;
     static constexpr int kTileBytes = kTileKeys * D * 2;  // a bf16 K or V tile
@@ -469,17 +482,19 @@ struct Layout {
     static constexpr int kQBytes = kPanels * kRows * 128;  // one query buffer
     static constexpr int kPBytes = kRows * kTileKeys * 2;  // one P buffer
     static constexpr int kStagesOff = 0;
-    static constexpr int kConvOff = kStages * kStageBytes;  // widened tiles, one set per stage
-    static constexpr int kQOff = kConvOff + kStages * kConvBytes;
+    static constexpr int kConvOff = kStages * kStageBytes;  // the ring of widened tiles
+    static constexpr int kQOff = kConvOff + kConvSlots * kConvBytes;
     static constexpr int kPOff = kQOff + 2 * kQBytes;
     static constexpr int kBarOff = kPOff + 2 * kPBytes;
     // barriers: full[kStages], empty[kStages], qfull[2], qempty[2], sready[2],
-    // sfree[2], pready[2], pvdone[2], drain, kready[kStages]
-    static constexpr int kNumBars = 2 * kStages + 13 + kStages;
+    // sfree[2], pready[2], pvdone[2], drain, cready[kConvSlots],
+    // kfree[kConvSlots], vfree[kConvSlots]
+    static constexpr int kNumBars = 2 * kStages + 13 + 3 * kConvSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
+    static_assert(kBytes <= 232448, "shared memory per CTA");
 };
 
 // K-major 128B-swizzled address of bf16 element (row, col) of a [64][64] panel
@@ -487,20 +502,20 @@ __device__ __forceinline__ uint32_t p_chunk_addr(uint32_t base, int row, int chu
     return base + row * 128 + ((chunk ^ (row & 7)) << 4);
 }
 
-// Two e4m3 values (element 0 in bits 0-7) -> bf16x2 (element 0 in the low
-// half): cvt to f16x2 (exact), each f16 to f32 (exact), and the upper half
-// of each f32 is the bf16 (exact: an e4m3 value has at most 4 significant
-// bits and a 4-bit exponent, well inside bf16).  NaN stays NaN.
-__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint32_t x) {
-    uint32_t h2, r;
-    asm("{\n .reg .b16 t;\n cvt.u16.u32 t, %1;\n cvt.rn.f16x2.e4m3x2 %0, t;\n}"
-        : "=r"(h2)
-        : "r"(x));
-    float lo, hi;
-    asm("{\n .reg .b16 a, b;\n mov.b32 {a, b}, %2;\n cvt.f32.f16 %0, a;\n cvt.f32.f16 %1, b;\n}"
-        : "=f"(lo), "=f"(hi)
-        : "r"(h2));
-    asm("prmt.b32 %0, %1, %2, 0x7632;" : "=r"(r) : "r"(__float_as_uint(lo)), "r"(__float_as_uint(hi)));
+// Two e4m3 codes, one in the low byte of each 16-bit half of u -> bf16x2.
+// Shifted into bf16 position (sign to bit 15, exponent field e and mantissa
+// m to bits 7..10 and 4..6) a code is the bf16 value 2^-120 times its e4m3
+// value: the exponent biases differ by 127 - 7, and an e4m3 subnormal
+// (e = 0) lands on a bf16 subnormal with the same 2^-120 factor.  One
+// multiply by 2^120 (exact: the product is representable) finishes the
+// conversion; a NaN code (e = 15, m = 7) first gets an all-ones exponent
+// field, so it stays NaN.  All full-rate integer and bf16x2 operations.
+__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint32_t u) {
+    const uint32_t mag = u & 0x007F007Fu;
+    const uint32_t nan = ((mag + 0x00010001u) & 0x00800080u) * 0xFFu;  // 0x7F80 where mag == 0x7F
+    const uint32_t bits = (mag << 4) | ((u & 0x00800080u) << 8) | nan;
+    uint32_t r;
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(bits), "r"(0x7B807B80u));  // 2^120
     return r;
 }
 
@@ -521,15 +536,18 @@ __device__ __forceinline__ void widen_tile(uint32_t src, uint32_t dst, int ct) {
                      : "r"(src + key * D + d0));
         const uint32_t row = dst + (d0 / 64) * 8192 + key * 128;
         const int j = (d0 % 64) / 8;  // the first of two 16-byte bf16 chunks
+        // bytes 0,1 / 2,3 of each word into the 16-bit halves of a register
+        auto lo = [](uint32_t w) { return __byte_perm(w, 0u, 0x4140); };
+        auto hi = [](uint32_t w) { return __byte_perm(w, 0u, 0x4342); };
         asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
                          row + ((j ^ (key & 7)) << 4)),
-                     "r"(e4m3x2_to_bf16x2(w0 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w0 >> 16)),
-                     "r"(e4m3x2_to_bf16x2(w1 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w1 >> 16))
+                     "r"(e4m3x2_to_bf16x2(lo(w0))), "r"(e4m3x2_to_bf16x2(hi(w0))),
+                     "r"(e4m3x2_to_bf16x2(lo(w1))), "r"(e4m3x2_to_bf16x2(hi(w1)))
                      : "memory");
         asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
                          row + (((j + 1) ^ (key & 7)) << 4)),
-                     "r"(e4m3x2_to_bf16x2(w2 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w2 >> 16)),
-                     "r"(e4m3x2_to_bf16x2(w3 & 0xffffu)), "r"(e4m3x2_to_bf16x2(w3 >> 16))
+                     "r"(e4m3x2_to_bf16x2(lo(w2))), "r"(e4m3x2_to_bf16x2(hi(w2))),
+                     "r"(e4m3x2_to_bf16x2(lo(w3))), "r"(e4m3x2_to_bf16x2(hi(w3)))
                      : "memory");
     }
 }
@@ -552,18 +570,32 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     const uint32_t b_full = bars, b_empty = bars + 8 * kStages, b_qfull = b_empty + 8 * kStages,
                    b_qempty = b_qfull + 16, b_sready = b_qempty + 16, b_sfree = b_sready + 16,
                    b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 16,
-                   b_kready = b_drain + 8;
-    // where the MMAs read stage s's bf16 K and V: the TMA tile, or the tile
-    // the conversion warps widened from e4m3
+                   b_cready = b_drain + 8, b_kfree = b_cready + 8 * Lt::kConvSlots,
+                   b_vfree = b_kfree + 8 * Lt::kConvSlots;
+    constexpr int kSlots = Lt::kConvSlots;
+    // where the MMAs read tile j's bf16 K and V (stage s = j % kStages): the
+    // TMA tile in the stage, or the ring slot j % kSlots the conversion warps
+    // widened it into
     const uint32_t kconv0 = sbase + Lt::kConvOff, vconv0 = kconv0 + (KF8 ? Lt::kTileBytes : 0);
-    auto k_src = [&](int st) {
-        return KF8 ? kconv0 + st * Lt::kConvBytes : sbase + st * Lt::kStageBytes;
+    auto k_src = [&](int st, long long j) {
+        return KF8 ? kconv0 + (int)(j % kSlots) * Lt::kConvBytes : sbase + st * Lt::kStageBytes;
     };
-    auto v_src = [&](int st) {
-        return VF8 ? vconv0 + st * Lt::kConvBytes : sbase + st * Lt::kStageBytes + Lt::kKBytes;
+    auto v_src = [&](int st, long long j) {
+        return VF8 ? vconv0 + (int)(j % kSlots) * Lt::kConvBytes
+                   : sbase + st * Lt::kStageBytes + Lt::kKBytes;
     };
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(sm + Lt::kMiscOff);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + Lt::kMiscOff + 4);
+    // a ring slot is written for tile j once the MMAs of tile j - kSlots that
+    // read it have completed (kfree after S, vfree after P V).  Only the
+    // conversion warps wait on kfree / vfree, and they wait for every tile in
+    // order: a parity wait is exact only when the barrier is at most one phase
+    // behind, which a thread that skipped tiles (the producer, which runs
+    // kStages tiles ahead of P V) could not ensure.
+    auto slot_free = [&](uint32_t bar, long long j) {
+        return j < kSlots || wait(bar + 8 * (int)(j % kSlots),
+                                  (uint32_t)(((j - kSlots) / kSlots) & 1), abort_flag, p.status);
+    };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
 
@@ -585,7 +617,11 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         mbar_init(b_pvdone + 8, 1);
         mbar_init(b_drain, 1);
         if (Lt::kConv)
-            for (int s = 0; s < kStages; ++s) mbar_init(b_kready + 8 * s, kConvWarps);
+            for (int c = 0; c < kSlots; ++c) {
+                mbar_init(b_cready + 8 * c, kConvWarps);
+                mbar_init(b_kfree + 8 * c, 1);
+                mbar_init(b_vfree + 8 * c, 1);
+            }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -619,6 +655,9 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     // an empty range (only when N < C) runs no loop below
     const long long ntiles = plan(p, lo, hi, w0) ? hi - lo : 0;
 
+    // the last loads each issuing thread started, for the abort path's drain
+    long long drain_tiles = 0, drain_copy = -1;
+    int drain_qseg = -1;
     if (warp == kProducerWarp) {
         // ================================ producer ===============================
         // Warp-uniform loop; one elected lane issues.  Stage s is reused once
@@ -628,6 +667,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
         Walk wl = w0;
         int qseg = -1;
+        long long issued = 0;  // tiles whose loads were issued (and a query segment's)
         bool ok = true;
         for (long long j = 0; j < ntiles && ok; ++j) {
             if (j == 0 || wl.t == 0) {  // the segment's query rows
@@ -674,18 +714,23 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                             tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
                                    p.value_slab, policy);
                     }
-                } else {  // the block's own K / V: bf16, straight to where the MMAs read
-                    mbar_arrive_expect_tx(full, 2 * Lt::kTileBytes);
+                } else {  // the block's own K / V (bf16): the operands read from the
+                          // stage; ring-slot operands are loaded by the conversion warps
+                    mbar_arrive_expect_tx(full, (KF8 ? 0 : Lt::kTileBytes) +
+                                                    (VF8 ? 0 : Lt::kTileBytes));
 #pragma unroll
                     for (int dp = 0; dp < Lt::kPanels; ++dp) {
-                        tma_4d(k_src(s) + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
-                        tma_4d(v_src(s) + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
+                        if (!KF8) tma_4d(kdst + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
+                        if (!VF8) tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
                     }
                 }
             }
             __syncwarp();
+            if (ok) issued = j + 1;
             walk_next(p, wl);
         }
+        drain_tiles = issued;
+        drain_qseg = qseg;
     } else if (warp == kMmaWarp) {
         // ================================== MMA ==================================
         const uint32_t id_s = idesc(kRows, kTileKeys, 0, 0);
@@ -693,11 +738,8 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         // descriptors are affine in the address: build each base once and add
         // (byte offset >> 4) for buffers and k-steps
         const uint64_t dq0 = sdesc(sbase + Lt::kQOff, 16, 1024);
-        const uint64_t dk0 = sdesc(k_src(0), 16, 1024);
-        const uint64_t dv0 = sdesc(v_src(0), 8192, 1024);
-        // byte distance between consecutive stages' K (V) tiles
-        constexpr int kKStride = KF8 ? Lt::kConvBytes : Lt::kStageBytes;
-        constexpr int kVStride = VF8 ? Lt::kConvBytes : Lt::kStageBytes;
+        const uint64_t dk0 = sdesc(k_src(0, 0), 16, 1024);
+        const uint64_t dv0 = sdesc(v_src(0, 0), 8192, 1024);
         const uint64_t dp0 = sdesc(sbase + Lt::kPOff, 16, 1024);
         Walk wsn = w0;  // walk of the next S
         int qseg = -1, qcur = 0;
@@ -710,9 +752,13 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                                 p.status);
             }
             const int s = (int)(kn % kStages);
-            // the stage's tiles in bf16: landed, and widened if stored as e4m3
-            ok = ok && wait((Lt::kConv ? b_kready : b_full) + 8 * s,
-                            (uint32_t)((kn / kStages) & 1), abort_flag, p.status);
+            // the tile's K and V in bf16: landed, and widened if stored as e4m3
+            if (Lt::kConv)
+                ok = ok && wait(b_cready + 8 * (int)(kn % kSlots), (uint32_t)((kn / kSlots) & 1),
+                                abort_flag, p.status);
+            else
+                ok = ok && wait(b_full + 8 * s, (uint32_t)((kn / kStages) & 1), abort_flag,
+                                p.status);
             if (kn >= 2)
                 ok = ok && wait(b_sfree + 8 * (int)(kn & 1), (uint32_t)(((kn - 2) >> 1) & 1),
                                 abort_flag, p.status);
@@ -721,7 +767,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 fence_after();
                 if (elect_one()) {
                     const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
-                    const uint64_t b0 = dk0 + (uint64_t)((s * kKStride) >> 4);
+                    const uint64_t b0 = dk0 + (uint64_t)((k_src(s, kn) - k_src(0, 0)) >> 4);
                     const uint32_t dS = tmem + (uint32_t)((kn & 1) * kTileKeys);
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
@@ -731,6 +777,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                         mma(dS, a0 + qoff, b0 + koff, id_s, kk > 0);
                     }
                     mma_commit(b_sready + 8 * (int)(kn & 1));
+                    if (KF8) mma_commit(b_kfree + 8 * (int)(kn % kSlots));
                     if (seg_end) mma_commit(b_qempty + 8 * qcur);
                 }
                 __syncwarp();
@@ -748,7 +795,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             if (elect_one()) {
                 const int s = (int)(k % kStages);
                 const uint64_t a0 = dp0 + (uint64_t)(((k & 1) * Lt::kPBytes) >> 4);
-                const uint64_t b0 = dv0 + (uint64_t)((s * kVStride) >> 4);
+                const uint64_t b0 = dv0 + (uint64_t)((v_src(s, k) - v_src(0, 0)) >> 4);
                 const uint32_t dO = tmem + 2 * kTileKeys;
 #pragma unroll
                 for (int kk = 0; kk < kTileKeys / 16; ++kk)
@@ -756,6 +803,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                         id_pv, (!first || kk > 0) ? 1u : 0u);
                 mma_commit(b_pvdone + 8 * (int)(k & 1));
                 mma_commit(b_empty + 8 * s);
+                if (VF8) mma_commit(b_vfree + 8 * (int)(k % kSlots));
             }
             __syncwarp();
             if (k + 2 < ntiles) next_s(k + 2);
@@ -770,23 +818,58 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         }
     } else if (Lt::kConv && warp >= kConvWarp0) {
         // ============================ e4m3 -> bf16 ===============================
-        // Widen every prefix tile's e4m3 K (and V) once it has landed, then
-        // release the stage to the MMA warp (kready); block tiles are bf16
-        // already and are only passed on.
+        // Widen every prefix tile's e4m3 K (and V) into its ring slot once it
+        // has landed and the slot is free, then hand the tile to the MMA warp
+        // (cready).  A block tile's K (V) is bf16 already: for a ring operand
+        // one elected lane of the first conversion warp loads it into the slot
+        // with a copy that completes on cready itself.
         const int ct = threadIdx.x - kConvWarp0 * 32;
         Walk wc = w0;
         bool ok = true;
         for (long long j = 0; j < ntiles && ok; ++j) {
             const int s = (int)(j % kStages);
+            const uint32_t cready = b_cready + 8 * (int)(j % kSlots);
             ok = wait(b_full + 8 * s, (uint32_t)((j / kStages) & 1), abort_flag, p.status);
             if (!ok) break;
-            if (wc.t < wc.nt - 1) {
-                if (KF8) widen_tile<D>(sbase + s * Lt::kStageBytes, k_src(s), ct);
-                if (VF8) widen_tile<D>(sbase + s * Lt::kStageBytes + Lt::kKBytes, v_src(s), ct);
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            if (wc.t == wc.nt - 1) {
+                if (KF8) ok = slot_free(b_kfree, j);
+                if (VF8) ok = ok && slot_free(b_vfree, j);
+                if (!ok) break;
+                if (warp == kConvWarp0) {
+                    if (elect_one()) {
+                        mbar_arrive_expect_tx(cready, ((KF8 ? 1 : 0) + (VF8 ? 1 : 0)) *
+                                                          Lt::kTileBytes);
+#pragma unroll
+                        for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                            if (KF8)
+                                tma_4d(k_src(s, j) + dp * 8192, &tm_kb, cready, dp * 64, wc.h, 0,
+                                       wc.b);
+                            if (VF8)
+                                tma_4d(v_src(s, j) + dp * 8192, &tm_vb, cready, dp * 64, wc.h, 0,
+                                       wc.b);
+                        }
+                    }
+                    drain_copy = j;
+                } else if (lane == 0) {
+                    mbar_arrive(cready);
+                }
+                __syncwarp();
+                walk_next(p, wc);
+                continue;
             }
+            if (KF8) {
+                ok = slot_free(b_kfree, j);
+                if (!ok) break;
+                widen_tile<D>(sbase + s * Lt::kStageBytes, k_src(s, j), ct);
+            }
+            if (VF8) {
+                ok = slot_free(b_vfree, j);
+                if (!ok) break;
+                widen_tile<D>(sbase + s * Lt::kStageBytes + Lt::kKBytes, v_src(s, j), ct);
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             __syncwarp();
-            if (lane == 0) mbar_arrive(b_kready + 8 * s);
+            if (lane == 0) mbar_arrive(cready);
             walk_next(p, wc);
         }
     } else {
@@ -923,7 +1006,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             l_sum += lt;
             // keys past the end of the tile may hold anything: zero their V rows
             if (nvalid < kTileKeys) {
-                const uint32_t vt = v_src(s);
+                const uint32_t vt = v_src(s, k);
                 const int nzero = (kTileKeys - nvalid) * 8 * Lt::kPanels;  // 16-byte chunks
                 for (int i = threadIdx.x; i < nzero; i += kSoftWarps * 32) {
                     const int panel = i / ((kTileKeys - nvalid) * 8);
@@ -1011,6 +1094,17 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     fence_before();
     __syncthreads();
     fence_after();
+    if (*abort_flag) {  // a wait gave up: copies still in flight land before exit
+        if (warp == kProducerWarp && elect_one()) {
+            for (long long j = drain_tiles - 1; j >= 0 && j >= drain_tiles - kStages; --j)
+                drain_wait(b_full + 8 * (int)(j % kStages), (uint32_t)((j / kStages) & 1));
+            for (int q = drain_qseg; q >= 0 && q >= drain_qseg - 1; --q)
+                drain_wait(b_qfull + 8 * (q & 1), (uint32_t)((q >> 1) & 1));
+        }
+        if (Lt::kConv && warp == kConvWarp0 && lane == 0 && drain_copy >= 0)
+            drain_wait(b_cready + 8 * (int)(drain_copy % kSlots),
+                       (uint32_t)((drain_copy / kSlots) & 1));
+    }
     if (warp == 0)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "n"(kTmemCols));

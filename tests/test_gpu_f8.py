@@ -29,9 +29,19 @@ def host_f8_cache(wl):
             synth.e4m3_codes(wl.seed, synth.T_VLOW, low))
 
 
-def run_f8(wl, kap, nu, layer=1, prefix=None, block=None, poison_tail=False, scale=0.0):
+def every_code(shape, shift):
+    """Codes cycling through all 254 finite e4m3 codes (subnormals included)."""
+    finite = np.array([c for c in range(256) if c not in (0x7F, 0xFF)], dtype=np.uint8)
+    n = int(np.prod(shape))
+    return finite[(np.arange(n) * 7 + shift) % finite.size].reshape(shape)
+
+
+def run_f8(wl, kap, nu, layer=1, prefix=None, block=None, poison_tail=False, scale=0.0,
+           all_codes=False, zero_q=False):
     import paper_2609_34538_gb300 as das
     kt, vt, kl, vl = host_f8_cache(wl)
+    if all_codes:
+        kl, vl = every_code(kl.shape, 0), every_code(vl.shape, 101)
     pl = wl.prefix_lens() if prefix is None else np.asarray(prefix, np.int32)
     bl = wl.block_lens() if block is None else np.asarray(block, np.int32)
     if poison_tail:  # positions past the prefix hold NaN: never read
@@ -41,6 +51,8 @@ def run_f8(wl, kap, nu, layer=1, prefix=None, block=None, poison_tail=False, sca
             kt[:, b, pl[b]:] = 0x7FC0
             vt[:, b, pl[b]:] = 0x7FC0
     q = wl_mod.gen_q(wl, layer)
+    if zero_q:
+        q = np.zeros_like(q)
     kb, vb = wl_mod.gen_block_kv(wl, layer)
     ref_o, ref_l = oracle.attention_f8(kt, vt, kl, vl, layer, kap, nu, pl, bl, q, kb, vb,
                                        scale=scale if scale > 0 else None)
@@ -78,6 +90,18 @@ def test_head_dims_e4m3(D):
 def test_nan_past_the_prefix_is_never_read_e4m3():
     run_f8(small(prefix=(300, 300)), 2, 6, prefix=[300, 129], block=[8, 3], poison_tail=True)
     run_f8(small(prefix=(300, 300)), 4, 4, prefix=[300, 129], block=[8, 3], poison_tail=True)
+
+
+def test_every_e4m3_code_is_widened_exactly():
+    """Keys and values that run through every finite code, subnormals and
+    +-448 included.  e4m3 keys are checked through the scores; e4m3 values
+    with zero queries, where every softmax weight is exactly 1 and each
+    output is the mean of the stored values (with random queries, values of
+    +-448 and random signs make the outputs small averages of large terms, and
+    the bf16 rounding of the weights, relative to the values, dominates)."""
+    run_f8(small(prefix=(1500, 1500)), 2, 6, all_codes=True)
+    for kap, nu in [(6, 3), (4, 4), (2, 6)]:
+        run_f8(small(prefix=(1500, 1500)), kap, nu, all_codes=True, zero_q=True)
 
 
 def test_split_across_many_ctas_e4m3():
