@@ -51,11 +51,13 @@ constexpr unsigned long long kWaitNs = 2000000000ull;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kSoftWarps = 4;
 constexpr int kProducerWarp = kSoftWarps;     // TMA loads
-constexpr int kMmaWarp = kSoftWarps + 1;      // tcgen05 MMAs
-constexpr int kConvWarp0 = kSoftWarps + 2;    // e4m3 -> bf16 widening (e4m3 variants)
+constexpr int kMmaWarp = kSoftWarps + 1;      // tcgen05 MMAs of P V
+constexpr int kSWarp = kSoftWarps + 2;        // tcgen05 MMAs of S
+constexpr int kConvWarp0 = kSoftWarps + 3;    // e4m3 -> bf16 widening (e4m3 variants)
 constexpr int kConvWarps = 4;
 constexpr int kRows = 64;            // M of every MMA (query rows per pair)
-constexpr int kTmemCols = 256;       // S buffers [0, 128), O [128, 128 + D)
+constexpr int kSBufs = 4;            // S buffers in tensor memory
+constexpr int kTmemCols = 512;       // S buffers [0, 64 kSBufs), O [64 kSBufs, 64 kSBufs + D)
 constexpr float kRescaleLog2 = 8.f;  // move the reference max only beyond 2^8
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -198,22 +200,27 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
-// 16 lanes x 2 halves: thread t < 16 gets lane t, columns [c, c + 16); thread
-// t + 16 gets lane t, columns [c + 32, c + 48).  With M = 64 a warp's rows sit
-// in its first 16 lanes, so two threads share each row.
-__device__ __forceinline__ void tmem_ld_half16(uint32_t taddr, float (&v)[16]) {
-    uint32_t r[16];
+// 32 columns of S for the calling thread (16 lanes x 2 halves): thread t < 16
+// of a warp gets TMEM lane t, columns [c, c + 32), thread t + 16 the same lane,
+// [c + 32, c + 64).  With M = 64 a warp's rows sit in its first 16 lanes, so
+// two threads share each row.
+__device__ __forceinline__ void tmem_ld_half32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
     asm volatile(
-        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
-        "%13,%14,%15}, [%16], 32;\n"
+        "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], "
+        "32;\n"
         "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
         : "r"(taddr)
         : "memory");
 #pragma unroll
-    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 // The O row of the calling thread's half: with M = 64, thread t < 16 of a warp
 // gets TMEM lane t, columns [64 g, 64 g + 32) for g < D / 64, and thread t + 16
@@ -464,14 +471,15 @@ __device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w)
 // 128-byte-swizzled layout the MMAs read, held in a ring of kConvSlots slots
 // (tile j in slot j % kConvSlots) rather than one per stage: the smaller
 // stages then fit 6 (or 7) deep instead of 4, which is what keeps more DRAM
-// requests in flight per SM.  A pair's block tile is bf16 and is loaded
-// straight into its ring slot (or, for bf16 operands, into the stage).
+// requests in flight per SM.  A pair's block tile is bf16: the conversion
+// warps load its e4m3-stored operands straight into the ring slot, the
+// producer the others into the stage.
 template <int D, bool KF8, bool VF8>
 struct Layout {
     static constexpr bool kConv = KF8 || VF8;
     static constexpr int kStages = (KF8 && VF8) ? 7 : kConv ? 6 : 4;
     static constexpr int kConvSlots = 2;
-    static constexpr int kThreads = (kSoftWarps + 2 + (kConv ? kConvWarps : 0)) * 32;
+    static constexpr int kThreads = (kSoftWarps + 3 + (kConv ? kConvWarps : 0)) * 32;
     static constexpr int kPanels = D / 64;
     static constexpr int kTileBytes = kTileKeys * D * 2;  // a bf16 K or V tile
     static constexpr int kTile8Bytes = kTileKeys * D;     // an e4m3 tile
@@ -486,10 +494,10 @@ struct Layout {
     static constexpr int kQOff = kConvOff + kConvSlots * kConvBytes;
     static constexpr int kPOff = kQOff + 2 * kQBytes;
     static constexpr int kBarOff = kPOff + 2 * kPBytes;
-    // barriers: full[kStages], empty[kStages], qfull[2], qempty[2], sready[2],
-    // sfree[2], pready[2], pvdone[2], drain, cready[kConvSlots],
-    // kfree[kConvSlots], vfree[kConvSlots]
-    static constexpr int kNumBars = 2 * kStages + 13 + 3 * kConvSlots;
+    // barriers: full[kStages], empty[kStages], qfull[2], qempty[2],
+    // sready[kSBufs], sfree[kSBufs], pready[2], pvdone[2], drain[2],
+    // cready[kConvSlots], kfree[kConvSlots], vfree[kConvSlots]
+    static constexpr int kNumBars = 2 * kStages + 10 + 2 * kSBufs + 3 * kConvSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
@@ -529,7 +537,14 @@ __device__ __forceinline__ void widen_tile(uint32_t src, uint32_t dst, int ct) {
 #pragma unroll
     for (int i = 0; i < kChunks / (kConvWarps * 32); ++i) {
         const int c = ct + i * kConvWarps * 32;
-        const int key = c / (D / 16), d0 = (c % (D / 16)) * 16;
+        // Chunk c: 16 elements jj of a 64-column panel of a key.  The 8 lanes
+        // of a quarter warp (one shared-memory wavefront of 16-byte accesses)
+        // take two keys of opposite parity, so their loads (rows of D bytes)
+        // and their swizzled stores each touch 8 distinct 16-byte bank groups.
+        const int jj = c & 3;
+        const int pnl = D == 128 ? (c >> 2) & 1 : 0;
+        const int key = D == 128 ? ((c >> 4) << 1) + (pnl ^ ((c >> 3) & 1)) : c >> 2;
+        const int d0 = pnl * 64 + jj * 16;
         uint32_t w0, w1, w2, w3;
         asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
                      : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
@@ -568,9 +583,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     const uint32_t sbase = smem_u32(sm);
     const uint32_t bars = sbase + Lt::kBarOff;
     const uint32_t b_full = bars, b_empty = bars + 8 * kStages, b_qfull = b_empty + 8 * kStages,
-                   b_qempty = b_qfull + 16, b_sready = b_qempty + 16, b_sfree = b_sready + 16,
-                   b_pready = b_sfree + 16, b_pvdone = b_pready + 16, b_drain = b_pvdone + 16,
-                   b_cready = b_drain + 8, b_kfree = b_cready + 8 * Lt::kConvSlots,
+                   b_qempty = b_qfull + 16, b_sready = b_qempty + 16,
+                   b_sfree = b_sready + 8 * kSBufs, b_pready = b_sfree + 8 * kSBufs,
+                   b_pvdone = b_pready + 16, b_drain = b_pvdone + 16,
+                   b_cready = b_drain + 16, b_kfree = b_cready + 8 * Lt::kConvSlots,
                    b_vfree = b_kfree + 8 * Lt::kConvSlots;
     constexpr int kSlots = Lt::kConvSlots;
     // where the MMAs read tile j's bf16 K and V (stage s = j % kStages): the
@@ -609,13 +625,16 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(b_qfull + 8 * i, 1);
             mbar_init(b_qempty + 8 * i, 1);
+            mbar_init(b_pready + 8 * i, kSoftWarps);
+        }
+        for (int i = 0; i < kSBufs; ++i) {
             mbar_init(b_sready + 8 * i, 1);
             mbar_init(b_sfree + 8 * i, kSoftWarps);
-            mbar_init(b_pready + 8 * i, kSoftWarps);
         }
         mbar_init(b_pvdone, 1);
         mbar_init(b_pvdone + 8, 1);
         mbar_init(b_drain, 1);
+        mbar_init(b_drain + 8, 1);
         if (Lt::kConv)
             for (int c = 0; c < kSlots; ++c) {
                 mbar_init(b_cready + 8 * c, kConvWarps);
@@ -731,8 +750,12 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         }
         drain_tiles = issued;
         drain_qseg = qseg;
-    } else if (warp == kMmaWarp) {
+    } else if (warp == kMmaWarp || warp == kSWarp) {
         // ================================== MMA ==================================
+        // Two issuing warps, each blocking on its own in-order stream: P V of
+        // tile k once its P is in shared memory (pready), and S of tile kn once
+        // its K has landed (or been widened), its segment's queries are in and
+        // TMEM buffer kn % kSBufs has been read by the softmax warps (sfree).
         const uint32_t id_s = idesc(kRows, kTileKeys, 0, 0);
         const uint32_t id_pv = idesc(kRows, D, 0, 1);
         // descriptors are affine in the address: build each base once and add
@@ -741,34 +764,36 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         const uint64_t dk0 = sdesc(k_src(0, 0), 16, 1024);
         const uint64_t dv0 = sdesc(v_src(0, 0), 8192, 1024);
         const uint64_t dp0 = sdesc(sbase + Lt::kPOff, 16, 1024);
-        Walk wsn = w0;  // walk of the next S
-        int qseg = -1, qcur = 0;
         bool ok = true;
-        auto next_s = [&](long long kn) {  // S of tile kn, two tiles ahead of P V
-            if (kn == 0 || wsn.t == 0) {
-                ++qseg;
-                qcur = qseg & 1;
-                ok = ok && wait(b_qfull + 8 * qcur, (uint32_t)((qseg >> 1) & 1), abort_flag,
-                                p.status);
-            }
-            const int s = (int)(kn % kStages);
-            // the tile's K and V in bf16: landed, and widened if stored as e4m3
-            if (Lt::kConv)
-                ok = ok && wait(b_cready + 8 * (int)(kn % kSlots), (uint32_t)((kn / kSlots) & 1),
-                                abort_flag, p.status);
-            else
-                ok = ok && wait(b_full + 8 * s, (uint32_t)((kn / kStages) & 1), abort_flag,
-                                p.status);
-            if (kn >= 2)
-                ok = ok && wait(b_sfree + 8 * (int)(kn & 1), (uint32_t)(((kn - 2) >> 1) & 1),
-                                abort_flag, p.status);
-            const bool seg_end = (wsn.t == wsn.nt - 1) || (kn + 1 == ntiles);
-            if (ok) {
+        if (warp == kSWarp) {
+            Walk wsn = w0;
+            int qseg = -1, qcur = 0;
+            for (long long kn = 0; kn < ntiles && ok; ++kn) {
+                if (kn == 0 || wsn.t == 0) {
+                    ++qseg;
+                    qcur = qseg & 1;
+                    ok = ok && wait(b_qfull + 8 * qcur, (uint32_t)((qseg >> 1) & 1), abort_flag,
+                                    p.status);
+                }
+                const int s = (int)(kn % kStages);
+                // the tile's K and V in bf16: landed, and widened if stored as e4m3
+                if (Lt::kConv)
+                    ok = ok && wait(b_cready + 8 * (int)(kn % kSlots),
+                                    (uint32_t)((kn / kSlots) & 1), abort_flag, p.status);
+                else
+                    ok = ok && wait(b_full + 8 * s, (uint32_t)((kn / kStages) & 1), abort_flag,
+                                    p.status);
+                if (kn >= kSBufs)
+                    ok = ok && wait(b_sfree + 8 * (int)(kn % kSBufs),
+                                    (uint32_t)(((kn - kSBufs) / kSBufs) & 1), abort_flag,
+                                    p.status);
+                if (!ok) break;
+                const bool seg_end = (wsn.t == wsn.nt - 1) || (kn + 1 == ntiles);
                 fence_after();
                 if (elect_one()) {
                     const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
                     const uint64_t b0 = dk0 + (uint64_t)((k_src(s, kn) - k_src(0, 0)) >> 4);
-                    const uint32_t dS = tmem + (uint32_t)((kn & 1) * kTileKeys);
+                    const uint32_t dS = tmem + (uint32_t)((kn % kSBufs) * kTileKeys);
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
                         // panel kk / 4, then 16 elements (32 bytes) within the 128-byte row
@@ -776,45 +801,46 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                         const uint32_t koff = ((kk >> 2) * 8192 + (kk & 3) * 32) >> 4;
                         mma(dS, a0 + qoff, b0 + koff, id_s, kk > 0);
                     }
-                    mma_commit(b_sready + 8 * (int)(kn & 1));
+                    mma_commit(b_sready + 8 * (int)(kn % kSBufs));
                     if (KF8) mma_commit(b_kfree + 8 * (int)(kn % kSlots));
                     if (seg_end) mma_commit(b_qempty + 8 * qcur);
                 }
                 __syncwarp();
+                walk_next(p, wsn);
             }
-            walk_next(p, wsn);
-        };
-        for (long long kn = 0; kn < 2 && kn < ntiles && ok; ++kn) next_s(kn);
-        Walk wm = w0;  // tile of the next P V
-        for (long long k = 0; k < ntiles && ok; ++k) {
-            const bool first = (k == 0) || (wm.t == 0);
-            ok = ok && wait(b_pready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1), abort_flag,
-                            p.status);
-            if (!ok) break;
-            fence_after();
-            if (elect_one()) {
-                const int s = (int)(k % kStages);
-                const uint64_t a0 = dp0 + (uint64_t)(((k & 1) * Lt::kPBytes) >> 4);
-                const uint64_t b0 = dv0 + (uint64_t)((v_src(s, k) - v_src(0, 0)) >> 4);
-                const uint32_t dO = tmem + 2 * kTileKeys;
+        } else {
+            Walk wm = w0;
+            for (long long k = 0; k < ntiles && ok; ++k) {
+                const bool first = (k == 0) || (wm.t == 0);
+                ok = wait(b_pready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1), abort_flag,
+                          p.status);
+                if (!ok) break;
+                fence_after();
+                if (elect_one()) {
+                    const int s = (int)(k % kStages);
+                    const uint64_t a0 = dp0 + (uint64_t)(((k & 1) * Lt::kPBytes) >> 4);
+                    const uint64_t b0 = dv0 + (uint64_t)((v_src(s, k) - v_src(0, 0)) >> 4);
+                    const uint32_t dO = tmem + kSBufs * kTileKeys;
 #pragma unroll
-                for (int kk = 0; kk < kTileKeys / 16; ++kk)
-                    mma(dO, a0 + (uint64_t)((kk * 32) >> 4), b0 + (uint64_t)((kk * 2048) >> 4),
-                        id_pv, (!first || kk > 0) ? 1u : 0u);
-                mma_commit(b_pvdone + 8 * (int)(k & 1));
-                mma_commit(b_empty + 8 * s);
-                if (VF8) mma_commit(b_vfree + 8 * (int)(k % kSlots));
+                    for (int kk = 0; kk < kTileKeys / 16; ++kk)
+                        mma(dO, a0 + (uint64_t)((kk * 32) >> 4),
+                            b0 + (uint64_t)((kk * 2048) >> 4), id_pv,
+                            (!first || kk > 0) ? 1u : 0u);
+                    mma_commit(b_pvdone + 8 * (int)(k & 1));
+                    mma_commit(b_empty + 8 * s);
+                    if (VF8) mma_commit(b_vfree + 8 * (int)(k % kSlots));
+                }
+                __syncwarp();
+                walk_next(p, wm);
             }
-            __syncwarp();
-            if (k + 2 < ntiles) next_s(k + 2);
-            walk_next(p, wm);
         }
-        // all MMAs issued here are complete before tensor memory is freed
+        // all MMAs this warp issued are complete before tensor memory is freed
         // (only a timed-out run can leave any in flight)
-        if (elect_one()) mma_commit(b_drain);
+        const uint32_t drain = b_drain + (warp == kSWarp ? 8 : 0);
+        if (elect_one()) mma_commit(drain);
         __syncwarp();
         const unsigned long long t0 = globaltimer();
-        while (!mbar_try_wait(b_drain, 0) && globaltimer() - t0 < kWaitNs) {
+        while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitNs) {
         }
     } else if (Lt::kConv && warp >= kConvWarp0) {
         // ============================ e4m3 -> bf16 ===============================
@@ -897,112 +923,95 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             }
             const int nvalid = block_tile ? ws.T : min(kTileKeys, ws.P - ws.t * kTileKeys);
             const int s = (int)(k % kStages);
-            // ---- scores: two compact passes over 16-column chunks of S ----
-            const bool ok_s = wait(b_sready + 8 * (int)(k & 1), (uint32_t)((k >> 1) & 1),
-                                   abort_flag, p.status);
+            // ---- scores of tile k ----
+            const bool ok_s = wait(b_sready + 8 * (int)(k % kSBufs),
+                                   (uint32_t)((k / kSBufs) & 1), abort_flag, p.status);
             fence_after();
-            const uint32_t s_addr = tmem + lane_base + (uint32_t)((k & 1) * kTileKeys);
+            const uint32_t s_addr = tmem + lane_base + (uint32_t)((k % kSBufs) * kTileKeys);
             const bool valid_row = row < rows_active && ok_s;
             // keys j < lim are visible to this row; a full prefix tile needs no
             // mask (rows of other lanes are computed but never stored)
             const int lim = !valid_row ? 0 : (block_tile ? min(nvalid, irow + 1) : nvalid);
             const bool full_tile = !block_tile && nvalid == kTileKeys;
             const float scale = p.scale_log2;
-            // first tile of a segment: the reference max comes from a max pass
-            if (first) {
-                float mt = -INFINITY;
-#pragma unroll 1
-                for (int c = 0; c < 32; c += 16) {
-                    float v[16];
-                    tmem_ld_half16(s_addr + c, v);
-                    const int key0 = half * 32 + c;
+            // The thread's 32 scores in registers (masked keys -> -inf); the
+            // row's tile max decides the reference first: the segment's first
+            // tile sets it, a later tile moves it (rescaling O and l) only when
+            // its max is beyond the reference by more than 2^8.
+            float v[32];
+            tmem_ld_half32(s_addr, v);
+            // the scores are in registers: S buffer k % kSBufs may take tile k + kSBufs
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_sfree + 8 * (int)(k % kSBufs));
+            const int key0 = half * 32;
+            if (!full_tile) {
 #pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        mt = fmaxf(mt, key0 + j < lim ? v[j] * scale : -INFINITY);
-                }
-                m_ref = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
+                for (int j = 0; j < 32; ++j) v[j] = key0 + j < lim ? v[j] * scale : -INFINITY;
             }
+            float mt;
+            {
+                float m16[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) m16[j] = fmaxf(v[j], v[j + 16]);
+#pragma unroll
+                for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+                    for (int j = 0; j < w; ++j) m16[j] = fmaxf(m16[j], m16[j + w]);
+                mt = full_tile ? m16[0] * scale : m16[0];
+            }
+            mt = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
+            if (first) {
+                m_ref = mt;
+            } else {
+                const bool jump = valid_row && mt > m_ref + kRescaleLog2;
+                if (__any_sync(kFull, jump)) {
+                    // O is stable once P V of tile k-1 is done
+                    wait(b_pvdone + 8 * (int)((k - 1) & 1), (uint32_t)(((k - 1) >> 1) & 1),
+                         abort_flag, p.status);
+                    fence_after();
+                    const float alpha = jump ? ex2(m_ref - mt) : 1.f;  // m_ref -inf gives 0
+                    if (jump) {
+                        m_ref = mt;
+                        l_sum *= alpha;
+                    }
+#pragma unroll 1
+                    for (int c = 0; c < D; c += 32) {
+                        float o[32];
+                        const uint32_t ta = tmem + lane_base + (uint32_t)(kSBufs * kTileKeys + c);
+                        tmem_ld32(ta, o);
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) o[j] *= alpha;
+                        tmem_st32(ta, o);
+                    }
+                }
+            }
+            // P = 2^(s - m) as bf16 into the swizzled P buffer (32 keys = 4 chunks)
+            const float mu = m_ref == -INFINITY ? 0.f : m_ref;
+            uint32_t w[16];
+            float l4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const float a = full_tile ? ex2(fmaf(v[2 * e], scale, -mu)) : ex2(v[2 * e] - mu);
+                const float b2 =
+                    full_tile ? ex2(fmaf(v[2 * e + 1], scale, -mu)) : ex2(v[2 * e + 1] - mu);
+                l4[e & 3] += a + b2;
+                w[e] = pack_bf16(a, b2);
+            }
+            const float lt = (l4[0] + l4[1]) + (l4[2] + l4[3]);
             // P buffer (k & 1) is free once P V of tile k-2, its last reader, is done
             // (pvdone[k & 1] completes once per P V of tiles with that parity)
             if (k >= 2) wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)(((k - 2) >> 1) & 1), abort_flag,
                              p.status);
             fence_after();
-            // P = 2^(s - m) as bf16 into the swizzled P buffer (16 keys = 2 chunks),
-            // with the tile max on the side; a second pass only if the max moved
-            // beyond the reference by more than 2^8
             const uint32_t pbuf = sbase + Lt::kPOff + (uint32_t)((k & 1) * Lt::kPBytes);
-            float lt = 0.f;
-#pragma unroll 1
-            for (int pass = 0; pass < 2; ++pass) {
-                const float mu = m_ref == -INFINITY ? 0.f : m_ref;
-                float mt = -INFINITY;
-                lt = 0.f;
-#pragma unroll 1
-                for (int c = 0; c < 32; c += 16) {
-                    float v[16];
-                    tmem_ld_half16(s_addr + c, v);
-                    const int key0 = half * 32 + c;
-                    uint32_t w[8];
-                    if (full_tile) {  // warp-uniform: no masks
-                        float vm = v[0];
 #pragma unroll
-                        for (int j = 1; j < 16; ++j) vm = fmaxf(vm, v[j]);
-                        mt = fmaxf(mt, vm * scale);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const float a = ex2(fmaf(v[2 * e], scale, -mu));
-                            const float b2 = ex2(fmaf(v[2 * e + 1], scale, -mu));
-                            lt += a + b2;
-                            w[e] = pack_bf16(a, b2);
-                        }
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const float x0 = key0 + 2 * e < lim ? v[2 * e] * scale : -INFINITY;
-                            const float x1 =
-                                key0 + 2 * e + 1 < lim ? v[2 * e + 1] * scale : -INFINITY;
-                            mt = fmaxf(mt, fmaxf(x0, x1));
-                            const float a = ex2(x0 - mu), b2 = ex2(x1 - mu);
-                            lt += a + b2;
-                            w[e] = pack_bf16(a, b2);
-                        }
-                    }
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                                     p_chunk_addr(pbuf, row, key0 / 8)),
-                                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
-                                 : "memory");
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                                     p_chunk_addr(pbuf, row, key0 / 8 + 1)),
-                                 "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
-                                 : "memory");
-                }
-                mt = fmaxf(mt, __shfl_xor_sync(kFull, mt, 16));
-                const bool jump = valid_row && !first && mt > m_ref + kRescaleLog2;
-                if (!__any_sync(kFull, jump)) break;
-                // O is stable once P V of tile k-1 is done
-                wait(b_pvdone + 8 * (int)((k - 1) & 1), (uint32_t)(((k - 1) >> 1) & 1), abort_flag,
-                     p.status);
-                fence_after();
-                // the max moved: rescale O and l to the new reference, redo P
-                const float alpha = jump ? ex2(m_ref - mt) : 1.f;  // m_ref -inf gives 0
-                if (jump) {
-                    m_ref = mt;
-                    l_sum *= alpha;
-                }
-#pragma unroll 1
-                for (int c = 0; c < D; c += 32) {
-                    float v[32];
-                    const uint32_t ta = tmem + lane_base + (uint32_t)(2 * kTileKeys + c);
-                    tmem_ld32(ta, v);
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] *= alpha;
-                    tmem_st32(ta, v);
-                }
-            }
-            // S of this tile is no longer read: its buffer may take tile k+2
-            fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(b_sfree + 8 * (int)(k & 1));
+            for (int q4 = 0; q4 < 4; ++q4)
+                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                 p_chunk_addr(pbuf, row, key0 / 8 + q4)),
+                             "r"(w[4 * q4]), "r"(w[4 * q4 + 1]), "r"(w[4 * q4 + 2]),
+                             "r"(w[4 * q4 + 3])
+                             : "memory");
             l_sum += lt;
             // keys past the end of the tile may hold anything: zero their V rows
             if (nvalid < kTileKeys) {
@@ -1039,7 +1048,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 const int gq = row % p.G;
                 // this thread's columns: [64 g + 32 half, +32) for each 64-column group g
                 float v[D / 2];
-                tmem_ld_orow<D>(tmem + lane_base + (uint32_t)(2 * kTileKeys), v);
+                tmem_ld_orow<D>(tmem + lane_base + (uint32_t)(kSBufs * kTileKeys), v);
                 if (write) {
                     uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
                                               (size_t)ws.h * p.G + gq) * D + 32 * half;
