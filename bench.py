@@ -318,7 +318,8 @@ def gpu_arm(args):
             "parallelism": "replicas" if world > 1 else "single GPU",
             "l2": "flushed before every timed step (512 MiB write)",
         },
-        "pct_of_hbm_peak": {"measured_copy_6663.9" if peak_kind == "measured" else "fallback":
+        "pct_of_hbm_peak": {(f"measured_copy_{peak:.1f}" if peak_kind == "measured"
+                             else f"fallback_{peak:.0f}"):
                             round(100 * gbs / world / peak, 1),
                             "nominal_8000": round(100 * gbs / world / 8000.0, 1)},
         "draft_tokens_per_s": round(world * tokens * K_steps / draft_s, 1),
