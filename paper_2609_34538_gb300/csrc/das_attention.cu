@@ -375,6 +375,13 @@ __device__ __forceinline__ Split split_from_total(const AttnParams &p, long long
     return sp;
 }
 
+// Clamped length read from L2 (not kept in L1, so that a value read before
+// the dependency wait can never be served stale to a later load).
+__device__ __forceinline__ int len_cg(const int32_t *a, int b, int cap) {
+    const int v = __ldcg(a + b);
+    return v < 0 ? 0 : (v > cap ? cap : v);
+}
+
 // Tiles of one pair of sequence b (0 past the batch); at most 2^25, so sums
 // over 32 sequences fit in 32 bits.
 __device__ __forceinline__ int seq_tiles(const AttnParams &p, int b) {
@@ -389,9 +396,17 @@ __device__ Split split_of(const AttnParams &p) {  // whole warp
     return split_from_total(p, total);
 }
 
+// a / b for 0 <= a, 0 < b: a 32-bit division when both fit (the usual case;
+// a 64-bit division is a long dependent instruction sequence).
+__device__ __forceinline__ long long udiv(long long a, long long b) {
+    if ((((unsigned long long)a | (unsigned long long)b) >> 32) == 0)
+        return (long long)((uint32_t)a / (uint32_t)b);
+    return a / b;
+}
+
 // The CTA whose weighted range holds weighted position q.
 __device__ __forceinline__ int cta_of_w(long long q, const Split &sp, int C) {
-    return (int)(((q + 1) * C - 1) / sp.W);
+    return (int)udiv((q + 1) * C - 1, sp.W);
 }
 
 // Range [lo, hi) of this CTA and the walk state of its first tile (a whole
@@ -399,16 +414,21 @@ __device__ __forceinline__ int cta_of_w(long long q, const Split &sp, int C) {
 // of the per-pair tile counts gives, for sequence b of a chunk, both the
 // tiles and the weighted positions before it; the tiles at the weighted
 // positions c W / C and (c+1) W / C are located in the same pass.
-__device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w) {
+// P0 / T0: the clamped lengths of sequence `lane` (0 past the batch), given
+// by the caller; with B <= 32 they are all the plan reads.
+__device__ bool plan(const AttnParams &p, int P0, int T0, long long &lo, long long &hi, Walk &w) {
     const int lane = threadIdx.x & 31;
-    const Split sp = split_of(p);
-    const long long lw = (long long)blockIdx.x * sp.W / p.num_ctas;
-    const long long hw = ((long long)blockIdx.x + 1) * sp.W / p.num_ctas;
+    const int nt0 = lane < p.B ? tiles_of(P0) : 0;
+    const Split sp =
+        p.B <= 32 ? split_from_total(p, (long long)__reduce_add_sync(kFull, (unsigned)nt0) * p.Hkv)
+                  : split_of(p);
+    const long long lw = udiv((long long)blockIdx.x * sp.W, p.num_ctas);
+    const long long hw = udiv(((long long)blockIdx.x + 1) * sp.W, p.num_ctas);
     lo = hi = sp.N;
     bool have_lo = false;
     long long run_w = 0, run_t = 0;  // weighted positions / tiles before the chunk
     for (int b0 = 0; b0 < p.B; b0 += 32) {
-        const int nt = seq_tiles(p, b0 + lane);
+        const int nt = b0 == 0 ? nt0 : seq_tiles(p, b0 + lane);
         int inc = nt;  // inclusive scan over the chunk
 #pragma unroll
         for (int d = 1; d < 32; d <<= 1) {
@@ -426,8 +446,8 @@ __device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w)
             const long long seq_w = run_w + ((long long)excl + (long long)sp.beta * f) * p.Hkv;
             const long long seq_t = run_t + (long long)excl * p.Hkv;
             const long long off = q - seq_w;
-            int h = (int)(off / (ntf + sp.beta));
-            int t = (int)(off % (ntf + sp.beta));
+            int h = (int)udiv(off, ntf + sp.beta);
+            int t = (int)(off - (long long)h * (ntf + sp.beta));
             if (t >= ntf) {  // inside a block tile's extra weight: the next pair
                 t = 0;
                 ++h;
@@ -436,7 +456,13 @@ __device__ bool plan(const AttnParams &p, long long &lo, long long &hi, Walk &w)
                 wk->b = b0 + f;
                 wk->h = h;
                 wk->t = t;
-                walk_load_seq(p, *wk);
+                if (b0 == 0) {  // lengths already in registers
+                    wk->P = __shfl_sync(kFull, P0, f);
+                    wk->T = __shfl_sync(kFull, T0, f);
+                    wk->nt = tiles_of(wk->P);
+                } else {
+                    walk_load_seq(p, *wk);
+                }
                 if (wk->h == p.Hkv) {
                     wk->h = 0;
                     ++wk->b;
@@ -661,18 +687,38 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     fence_after();
     const uint32_t tmem = *tmem_slot;
 
+    // The plan from the lengths as they read before the dependency wait (a
+    // kernel before this one may still change them); after the wait they are
+    // read again and the plan is kept only if every length is unchanged.
+    const int lane0 = threadIdx.x & 31;
+    const bool spec = p.B <= 32;
+    long long lo = 0, hi = 0, ntiles = 0;
+    Walk w0 = {0, 0, 0, 1, 0, 0};
+    int sP = 0, sT = 0;
+    if (spec) {
+        sP = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
+        sT = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
+        ntiles = plan(p, sP, sT, lo, hi, w0) ? hi - lo : 0;
+    }
+
     // every input (and the workspace) may be written by the previous kernel
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    {
+        const int P1 = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
+        const int T1 = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
+        if (!(spec && __all_sync(kFull, P1 == sP && T1 == sT))) {
+            lo = hi = 0;
+            w0 = {0, 0, 0, 1, 0, 0};
+            ntiles = plan(p, P1, T1, lo, hi, w0) ? hi - lo : 0;
+        }
+    }
 
     if (blockIdx.x == 0 && threadIdx.x == 0)
         for (int b = 0; b < p.B; ++b)
             if (p.prefix_len[b] != clamp_prefix(p, b) || p.block_len[b] != clamp_block(p, b))
                 atomicOr(p.status, kStatusClamped);
-    long long lo, hi;
-    Walk w0 = {0, 0, 0, 1, 0, 0};
     // an empty range (only when N < C) runs no loop below
-    const long long ntiles = plan(p, lo, hi, w0) ? hi - lo : 0;
 
     // the last loads each issuing thread started, for the abort path's drain
     long long drain_tiles = 0, drain_copy = -1;
