@@ -6,7 +6,7 @@ import torch
 import oracle
 import synth
 from synth import workloads as wl_mod
-from tests.gpu_util import dev_bf16, dev_i32, host_bits
+from tests.gpu_util import assert_close, dev_bf16, dev_i32, host_bits
 
 pytestmark = pytest.mark.gpu
 
@@ -115,3 +115,47 @@ def test_verify_accept_append_chain_on_device():
     assert np.array_equal(acc.cpu().numpy(), a_star)
     assert np.array_equal(host_bits(cache.k), K2) and np.array_equal(host_bits(cache.v), V2)
     assert np.array_equal(pl.cpu().numpy(), pl2) and int(flag.item()) == f2 == 0
+
+
+def test_attention_right_after_append_sees_the_new_lengths():
+    """append -> attention -> append -> ... in one stream with no host round
+    trip: each attention call plans its split from prefix_len, which the
+    append just before it bumps on the device, and must attend over exactly
+    the updated prefix (the cached rows the append wrote included)."""
+    import paper_2609_34538_gb300 as das
+    rounds = 6
+    wl = wl_mod.WORKLOADS["verify"].replace(batch=3, layers=1, depths=2, key_depth=2,
+                                            value_depth=2, prefix=(90, 200), vocab=500)
+    W = wl.max_block
+    wl = wl.replace(extra_capacity=rounds * W)
+    pl0 = np.array([90, 130, 200], dtype=np.int32)
+    K, V = wl_mod.gen_cache(wl, depths=range(1, wl.depths + 1), tokens=int(pl0.max()))
+    kn, vn = wl_mod.gen_staged(wl, W)
+    rng = np.random.default_rng(11)
+    accs = rng.integers(0, W + 1, size=(rounds, wl.batch)).astype(np.int32)
+    cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+    ws = das.new_workspace(cache, wl.q_heads, W)
+    pl, bl = dev_i32(pl0), dev_i32(wl.block_lens())
+    q = dev_bf16(wl_mod.gen_q(wl, 0))
+    kb, vb = map(dev_bf16, wl_mod.gen_block_kv(wl, 0))
+    kn_d, vn_d = dev_bf16(kn), dev_bf16(vn)
+    acc_d = torch.from_numpy(accs).cuda()
+    flag = torch.zeros(1, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    outs = []
+    for i in range(rounds):
+        das.das_kv_append(cache, kn_d, vn_d, acc_d[i], pl, flag)
+        o, l = das.das_verify_attention(cache, 0, wl.depths, pl, bl, q, kb, vb, ws)
+        outs.append((o, l))
+    torch.cuda.synchronize()
+    assert int(flag.item()) == 0 and das.workspace_status(ws) == 0
+    Kh, Vh, plh = K, V, pl0
+    for i in range(rounds):
+        Kh, Vh, plh, f = oracle.kv_append(Kh, Vh, kn, vn, accs[i], plh)
+        assert f == 0
+        ref_o, ref_l = oracle.attention(Kh, Vh, 0, wl.depths, wl.depths, plh, wl.block_lens(),
+                                        wl_mod.gen_q(wl, 0), *wl_mod.gen_block_kv(wl, 0))
+        o, l = outs[i]
+        assert_close(o.float().cpu().numpy(), ref_o, l.cpu().numpy(), ref_l,
+                     where=f"[round {i} prefix {plh.tolist()}]")
+    assert np.array_equal(pl.cpu().numpy(), plh)
