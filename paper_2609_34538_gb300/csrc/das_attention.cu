@@ -57,6 +57,7 @@ constexpr int kConvWarp0 = kSoftWarps + 3;    // e4m3 -> bf16 widening (e4m3 var
 constexpr int kConvWarps = 4;
 constexpr int kRows = 64;            // M of every MMA (query rows per pair)
 constexpr int kSBufs = 4;            // S buffers in tensor memory
+constexpr int kPrefetchTiles = 2;    // prefix tiles pulled into L2 before the dependency wait
 constexpr int kTmemCols = 512;       // S buffers [0, 64 kSBufs), O [64 kSBufs, 64 kSBufs + D)
 constexpr float kRescaleLog2 = 8.f;  // move the reference max only beyond 2^8
 
@@ -130,6 +131,14 @@ __device__ __forceinline__ void tma_5d(uint32_t dst, const CUtensorMap *map, uin
         "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
         "r"(c4), "l"(policy)
         : "memory");
+}
+// L2 prefetch of one box (no shared memory, no barrier).
+__device__ __forceinline__ void tma_prefetch_5d(const CUtensorMap *map, int c0, int c1, int c2,
+                                                int c3, int c4) {
+    asm volatile("cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+                 : "memory");
 }
 __device__ __forceinline__ void tma_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
                                        int c1, int c2, int c3) {
@@ -699,6 +708,22 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         sP = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
         sT = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
         ntiles = plan(p, sP, sT, lo, hi, w0) ? hi - lo : 0;
+        // While the kernels before this one finish, pull the range's first
+        // prefix tiles into L2 (the cache is L2-coherent: if a kernel before
+        // this one writes them, the loads after the wait still see its data).
+        if (warp == kProducerWarp && elect_one()) {
+            Walk wp = w0;
+            for (long long j = 0; j < ntiles && j < kPrefetchTiles && wp.t < wp.nt - 1; ++j) {
+                const int tok = wp.t * kTileKeys;
+#pragma unroll
+                for (int dp = 0; dp < (KF8 ? 1 : Lt::kPanels); ++dp)
+                    tma_prefetch_5d(&tm_k, dp * 64, wp.h, tok, wp.b, p.key_slab);
+#pragma unroll
+                for (int dp = 0; dp < (VF8 ? 1 : Lt::kPanels); ++dp)
+                    tma_prefetch_5d(&tm_v, dp * 64, wp.h, tok, wp.b, p.value_slab);
+                ++wp.t;  // stays inside the pair: its last (block) tile ends the loop
+            }
+        }
     }
 
     // every input (and the workspace) may be written by the previous kernel
