@@ -11,31 +11,37 @@
 // launched right after as a programmatic dependent, combines each split
 // pair's partials by log-sum-exp.
 //
-// One CTA = four softmax warps + one TMA warp + one MMA warp.
-//   producer (warp 4): TMA loads of 64-key K and V tiles STAGES ahead into a
+// One CTA = four softmax warps + one TMA warp + two MMA warps (+ four
+// conversion warps when prefix keys or values are stored as e4m3).
+//   producer (warp 4): TMA loads of 64-key K and V tiles kStages ahead into a
 //     ring of shared-memory stages, and of each segment's query rows (the
 //     pair's G * max_block rows, ordered i * G + g, which is the order of a
 //     {64, G, max_block} box).
-//   MMA (warp 5, one elected lane issues):
-//       S = Q K^T    tcgen05.mma M=64 N=64 K=D   -> S buffer (k % 2) in TMEM
+//   P V issuer (warp 5) and S issuer (warp 6), one elected lane each, each
+//   blocking on its own in-order barriers:
+//       S = Q K^T    tcgen05.mma M=64 N=64 K=D   -> S buffer (k % 4) in TMEM
 //       O += P V     tcgen05.mma M=64 N=D K=64   -> O in TMEM
-//     S of tile k+2 is issued right after P V of tile k, so the tensor core
-//     works ahead while the softmax warps handle the current tile.  A stage is
-//     refilled once the P V that read it has completed.
+//     S of tile k is issued once its K has landed (or been widened) and the
+//     softmax warps have read S buffer k % 4, so the tensor core runs up to
+//     four tiles ahead of the softmax.  A stage is refilled once the P V that
+//     read it has completed.
 //   softmax warps: an M=64 MMA puts row r in TMEM lane 32 (r / 16) + r % 16, so
 //     warp w owns rows 16w..16w+15 and two threads share a row (one per half
-//     of the 64 keys).  They load the row's scores, mask and scale them (base
-//     2), keep a reference max m that only moves when a score exceeds it by
-//     more than 2^8 (then O and l are rescaled in TMEM), write P = 2^(s - m)
-//     as bf16 into a 128-byte-swizzled [64 rows][64 keys] buffer (the K-major
-//     A operand of P V) and accumulate l.  At the end of a segment they read
-//     the O rows from TMEM and write O / l and the lse (or the partial).
+//     of the 64 keys).  They load the row's scores (and free the S buffer),
+//     mask and scale them (base 2), keep a reference max m that only moves
+//     when a score exceeds it by more than 2^8 (then O and l are rescaled in
+//     TMEM), write P = 2^(s - m) as bf16 into a 128-byte-swizzled [64 rows]
+//     [64 keys] buffer (the K-major A operand of P V) and accumulate l.  At
+//     the end of a segment they read the O rows from TMEM and write O / l and
+//     the lse (or the partial).
 // The kernel is launched as a programmatic dependent of the previous kernel
-// in the stream: barrier set-up and the tensor-memory allocation overlap the
-// previous kernel's tail, and nothing global is read or written before
+// in the stream: barrier set-up, the tensor-memory allocation, the work plan
+// (from lengths read before the wait, checked again after it) and an L2
+// prefetch of the first tiles overlap the previous kernel's tail; nothing
+// global is written, and nothing read is used unchecked, before
 // griddepcontrol.wait.  Every wait is bounded (2 s); a time-out sets the
-// status word and stops the CTA's waits.  Tensor memory (256 columns) is freed
-// before the CTA exits.
+// status word and stops the CTA's waits.  Tensor memory (512 columns) is
+// freed before the CTA exits.
 #include <cuda_bf16.h>
 
 #include <atomic>
@@ -751,7 +757,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     if (warp == kProducerWarp) {
         // ================================ producer ===============================
         // Warp-uniform loop; one elected lane issues.  Stage s is reused once
-        // the P V that read it has completed (the MMA warp commits empty[s]);
+        // the P V that read it has completed (the P V warp commits empty[s]);
         // a query buffer once the last S of the segment before last completed.
         uint64_t policy;
         asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
@@ -916,7 +922,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     } else if (Lt::kConv && warp >= kConvWarp0) {
         // ============================ e4m3 -> bf16 ===============================
         // Widen every prefix tile's e4m3 K (and V) into its ring slot once it
-        // has landed and the slot is free, then hand the tile to the MMA warp
+        // has landed and the slot is free, then hand the tile to the S warp
         // (cready).  A block tile's K (V) is bf16 already: for a ring operand
         // one elected lane of the first conversion warp loads it into the slot
         // with a copy that completes on cready itself.
