@@ -551,20 +551,21 @@ __device__ __forceinline__ uint32_t p_chunk_addr(uint32_t base, int row, int chu
     return base + row * 128 + ((chunk ^ (row & 7)) << 4);
 }
 
-// Two e4m3 codes, one in the low byte of each 16-bit half of u -> bf16x2.
-// Shifted into bf16 position (sign to bit 15, exponent field e and mantissa
-// m to bits 7..10 and 4..6) a code is the bf16 value 2^-120 times its e4m3
-// value: the exponent biases differ by 127 - 7, and an e4m3 subnormal
-// (e = 0) lands on a bf16 subnormal with the same 2^-120 factor.  One
-// multiply by 2^120 (exact: the product is representable) finishes the
-// conversion; a NaN code (e = 15, m = 7) first gets an all-ones exponent
-// field, so it stays NaN.  All full-rate integer and bf16x2 operations.
-__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint32_t u) {
-    const uint32_t mag = u & 0x007F007Fu;
-    const uint32_t nan = ((mag + 0x00010001u) & 0x00800080u) * 0xFFu;  // 0x7F80 where mag == 0x7F
-    const uint32_t bits = (mag << 4) | ((u & 0x00800080u) << 8) | nan;
+// Two e4m3 codes (the low and high byte of a) -> bf16x2 (low, high half):
+// the hardware conversion to f16x2 (exact: every e4m3 value, NaN included, is
+// an f16 value), each half widened to f32 and the pair rounded to bf16x2
+// (exact again: an e4m3 value has at most 4 significant bits).
+__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint32_t a) {
+    uint32_t h;
+    asm("{\n .reg .b16 t;\n cvt.u16.u32 t, %1;\n cvt.rn.f16x2.e4m3x2 %0, t;\n}\n"
+        : "=r"(h)
+        : "r"(a));
+    float f0, f1;
+    asm("{\n .reg .b16 l, u;\n mov.b32 {l, u}, %2;\n cvt.f32.f16 %0, l;\n cvt.f32.f16 %1, u;\n}\n"
+        : "=f"(f0), "=f"(f1)
+        : "r"(h));
     uint32_t r;
-    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(bits), "r"(0x7B807B80u));  // 2^120
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(f1), "f"(f0));
     return r;
 }
 
@@ -593,8 +594,8 @@ __device__ __forceinline__ void widen_tile(uint32_t src, uint32_t dst, int ct) {
         const uint32_t row = dst + (d0 / 64) * 8192 + key * 128;
         const int j = (d0 % 64) / 8;  // the first of two 16-byte bf16 chunks
         // bytes 0,1 / 2,3 of each word into the 16-bit halves of a register
-        auto lo = [](uint32_t w) { return __byte_perm(w, 0u, 0x4140); };
-        auto hi = [](uint32_t w) { return __byte_perm(w, 0u, 0x4342); };
+        auto lo = [](uint32_t w) { return w & 0xFFFFu; };
+        auto hi = [](uint32_t w) { return w >> 16; };
         asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
                          row + ((j ^ (key & 7)) << 4)),
                      "r"(e4m3x2_to_bf16x2(lo(w0))), "r"(e4m3x2_to_bf16x2(hi(w0))),
