@@ -48,6 +48,20 @@ def test_ragged_batch_with_empty_rows():
     run_small(wl, prefix=[0, 1, 600, 64, 333, 0], block=[16, 0, 3, 8, 1, 0])
 
 
+@pytest.mark.parametrize("B", [33, 70])
+def test_more_than_32_sequences(B):
+    """Batches past one warp's 32 lanes: the split is planned after the
+    dependency wait over several 32-sequence chunks, and walks cross from one
+    chunk's sequences into the next; ragged lengths including P = 0 and T = 0."""
+    rng = np.random.default_rng(B)
+    prefix = rng.integers(0, 300, size=B).astype(np.int32)
+    block = rng.integers(0, 9, size=B).astype(np.int32)
+    prefix[::7] = 0
+    block[::11] = 0
+    wl = small(batch=B, q_heads=4, kv_heads=2, head_dim=64, prefix=(0, 300), block=(8,))
+    run_small(wl, prefix=prefix, block=block)
+
+
 def test_split_across_many_ctas():
     """More tiles than CTAs for one pair: hundreds of partials merged."""
     run_small(small(batch=1, kv_heads=1, q_heads=4, prefix=(20000, 20000), block=(16,)))
