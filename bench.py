@@ -50,6 +50,10 @@ def parse():
                     help="skip the long-prefix draft-phase measurements")
     ap.add_argument("--layers", type=int, default=0,
                     help="override the workload's layer count (smaller profiling captures)")
+    ap.add_argument("--probe", default="",
+                    help="run only one probe (draft:long, draft:batched, e4m3:decode, "
+                         "e4m3:long) with --steps/--warmup/--layers and print its result: "
+                         "for profiling captures")
     ap.add_argument("--compact-depths", action="store_true",
                     help="store 2 depths (key depth 1, value depth 2) instead of R: the same "
                          "bytes per call in a smaller cache, for profiling captures")
@@ -156,6 +160,15 @@ def gpu_arm(args):
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     dev = torch.device("cuda", local)
+    if args.probe:  # one probe alone (profiling captures); no benchmark line
+        kind, _, name = args.probe.partition(":")
+        fn = {"draft": draft_probe, "e4m3": f8_probe}.get(kind)
+        if fn is None or name not in wlm.WORKLOADS:
+            raise SystemExit(f"bench: unknown probe {args.probe!r}")
+        peak, _ = peaks()
+        print(json.dumps({"probe": args.probe, **fn(name, dev, args.steps, args.warmup, peak,
+                                                     layers=args.layers)}))
+        return
     wl = wlm.WORKLOADS[args.workload]
     if args.layers:
         wl = wl.replace(layers=args.layers)
@@ -347,7 +360,7 @@ def gpu_arm(args):
         dist.destroy_process_group()
 
 
-def draft_probe(name, dev, steps, warmup, peak):
+def draft_probe(name, dev, steps, warmup, peak, layers=0):
     """Per-call time of another workload's draft phase, timed like the main
     one (a CUDA graph of its L layer calls, L2 flushed before every replay).
     Only the two depth slabs the calls read are stored (depths compacted to
@@ -359,6 +372,8 @@ def draft_probe(name, dev, steps, warmup, peak):
     from synth import workloads as wlm
 
     wl = wlm.WORKLOADS[name].replace(depths=2, key_depth=1, value_depth=2)
+    if layers:
+        wl = wl.replace(layers=layers)
     L, B, W = wl.layers, wl.batch, wl.max_block
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
@@ -406,7 +421,7 @@ def draft_probe(name, dev, steps, warmup, peak):
             "pct_of_nominal_8000": round(100 * gbs / 8000.0, 1), "steps": len(ms)}
 
 
-def f8_probe(name, dev, steps, warmup, peak):
+def f8_probe(name, dev, steps, warmup, peak, layers=0):
     """Mature-V draft phase of workload `name` on the e4m3 cache variant
     (keys at depth r stored as e4m3, values at depth R as bf16; not in the
     paper), timed like the bf16 probes; bytes per call count 1 byte per key
@@ -418,6 +433,8 @@ def f8_probe(name, dev, steps, warmup, peak):
     from synth import workloads as wlm
 
     wl = wlm.WORKLOADS[name].replace(depths=2, key_depth=1, value_depth=2)
+    if layers:
+        wl = wl.replace(layers=layers)
     L, B, W = wl.layers, wl.batch, wl.max_block
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
