@@ -60,6 +60,24 @@ def parse():
     return ap.parse_args()
 
 
+def max_over_ranks(values, world, device):
+    """Each timing value as the maximum over the ranks (the slowest replica
+    sets the whole job's time); the values of this rank when world == 1."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def whole_job_gbs(world, bytes_per_step, steps, seconds):
+    """Whole-job throughput: the bytes all ranks processed (each rank a full
+    replica of the workload) over the slowest rank's time."""
+    return world * bytes_per_step * steps / seconds / 1e9
+
+
 def dist_env():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
             int(os.environ.get("LOCAL_RANK", 0)))
@@ -272,12 +290,9 @@ def gpu_arm(args):
     draft_bytes = wl.prefix_bytes_per_layer() * L
     verify_bytes = wlv.prefix_bytes_per_layer() * L
     draft_s = sum(draft_ms) / 1e3
-    totals = torch.tensor([draft_s, sum(step_ms) / 1e3], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(totals, op=dist.ReduceOp.MAX)
-    draft_s, step_s = totals.tolist()
+    draft_s, step_s = max_over_ranks([draft_s, sum(step_ms) / 1e3], world, dev)
     K_steps = args.steps
-    gbs = world * draft_bytes * K_steps / draft_s / 1e9
+    gbs = whole_job_gbs(world, draft_bytes, K_steps, draft_s)
     tokens = int(wl.block_lens().sum())
     peak, peak_kind = peaks()
     per_launch_ms = statistics.mean(draft_ms) / L
@@ -286,9 +301,8 @@ def gpu_arm(args):
 
     e2e = None if args.no_e2e else e2e_arm(args, wl, cache, pl, P0, bl, ws, stream, dev)
     if e2e is not None and world > 1:
-        t = torch.tensor([e2e.pop("_seconds")], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e["value"] = world * draft_bytes * K_steps / t.item() / 1e9
+        (t,) = max_over_ranks([e2e.pop("_seconds")], world, dev)
+        e2e["value"] = whole_job_gbs(world, draft_bytes, K_steps, t)
     elif e2e is not None:
         e2e.pop("_seconds")
 
