@@ -540,7 +540,8 @@ struct Layout {
     // cready[kConvSlots], kfree[kConvSlots], vfree[kConvSlots]
     static constexpr int kNumBars = 2 * kStages + 10 + 2 * kSBufs + 3 * kConvSlots;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
-    static constexpr int kBytes = kMiscOff + 16 + 1024;  // + alignment slack
+    static constexpr int kLenOff = kMiscOff + 16;  // lengths read before the dependency wait
+    static constexpr int kBytes = kLenOff + 64 * 4 + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
     static_assert(kBytes <= 232448, "shared memory per CTA");
@@ -659,7 +660,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
 
     // set-up that touches no global memory: it may overlap the previous
     // kernel in the stream (programmatic dependent launch)
-    if (threadIdx.x == 0) {
+    auto init_bars = [&]() {  // one thread
         for (int s = 0; s < kStages; ++s) {
             mbar_init(b_full + 8 * s, 1);
             mbar_init(b_empty + 8 * s, 1);
@@ -683,8 +684,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 mbar_init(b_kfree + 8 * c, 1);
                 mbar_init(b_vfree + 8 * c, 1);
             }
-        *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    };
+    int *len_sm = reinterpret_cast<int *>(sm + Lt::kLenOff);  // [0, 32) P, [32, 64) T
+    const int lane0 = threadIdx.x & 31;
+    const bool spec = p.B <= 32;
+    if (threadIdx.x == 0) {
+        init_bars();
+        *abort_flag = 0;
     }
     if (warp == 0) {
         asm volatile(
@@ -692,6 +699,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 smem_u32(const_cast<uint32_t *>(tmem_slot))),
             "n"(kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    // The lengths as they read before the dependency wait (a kernel before
+    // this one may still change them), one copy for the whole CTA: every
+    // warp plans from the same values, and the check after the wait is the
+    // same in every warp.
+    if (spec && warp == kProducerWarp) {
+        len_sm[lane0] = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
+        len_sm[32 + lane0] = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
     }
     if (warp == kProducerWarp && elect_one()) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
@@ -703,17 +718,15 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    // The plan from the lengths as they read before the dependency wait (a
-    // kernel before this one may still change them); after the wait they are
-    // read again and the plan is kept only if every length is unchanged.
-    const int lane0 = threadIdx.x & 31;
-    const bool spec = p.B <= 32;
+    // The plan from the lengths as they read before the dependency wait;
+    // after the wait they are read again and the plan is kept only if every
+    // length is unchanged.
     long long lo = 0, hi = 0, ntiles = 0;
     Walk w0 = {0, 0, 0, 1, 0, 0};
     int sP = 0, sT = 0;
     if (spec) {
-        sP = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
-        sT = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
+        sP = len_sm[lane0];
+        sT = len_sm[32 + lane0];
         ntiles = plan(p, sP, sT, lo, hi, w0) ? hi - lo : 0;
         // While the kernels before this one finish, pull the range's first
         // prefix tiles into L2 (the cache is L2-coherent: if a kernel before
@@ -733,16 +746,106 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         }
     }
 
+    // Producer state and one step of its loop (tile j of the range): the
+    // first steps may run before the lengths are checked (below).
+    Walk wl = w0;
+    int qseg = -1;
+    long long issued = 0, j = 0;  // tiles whose loads were issued; next tile
+    bool ok = true;
+    uint64_t policy = 0;
+    if (warp == kProducerWarp)
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+    auto produce = [&]() {
+        if (j == 0 || wl.t == 0) {  // the segment's query rows
+            ++qseg;
+            const int qb = qseg & 1;
+            if (qseg >= 2)
+                ok = ok && wait(b_qempty + 8 * qb, (uint32_t)(((qseg - 2) >> 1) & 1),
+                                abort_flag, p.status);
+            if (ok && elect_one()) {
+                const uint32_t full = b_qfull + 8 * qb;
+                const uint32_t dst = sbase + Lt::kQOff + qb * Lt::kQBytes;
+                mbar_arrive_expect_tx(full, Lt::kPanels * p.rows_max * 128);
+#pragma unroll
+                for (int dp = 0; dp < Lt::kPanels; ++dp)
+                    tma_4d(dst + dp * (kRows * 128), &tm_q, full, dp * 64, wl.h * p.G, 0,
+                           wl.b);
+            }
+        }
+        const int s = (int)(j % kStages);
+        if (j >= kStages)
+            ok = ok && wait(b_empty + 8 * s, (uint32_t)(((j - kStages) / kStages) & 1),
+                            abort_flag, p.status);
+        if (ok && elect_one()) {
+            const uint32_t full = b_full + 8 * s;
+            const uint32_t kdst = sbase + Lt::kStagesOff + s * Lt::kStageBytes;
+            const uint32_t vdst = kdst + Lt::kKBytes;
+            if (wl.t < wl.nt - 1) {
+                const int tok = wl.t * kTileKeys;
+                mbar_arrive_expect_tx(full, Lt::kStageBytes);
+                // an e4m3 tile is one {D, 1, 64} box, a bf16 tile D / 64 swizzled panels
+                if (KF8) {
+                    tma_5d(kdst, &tm_k, full, 0, wl.h, tok, wl.b, p.key_slab, policy);
+                } else {
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp)
+                        tma_5d(kdst + dp * 8192, &tm_k, full, dp * 64, wl.h, tok, wl.b,
+                               p.key_slab, policy);
+                }
+                if (VF8) {
+                    tma_5d(vdst, &tm_v, full, 0, wl.h, tok, wl.b, p.value_slab, policy);
+                } else {
+#pragma unroll
+                    for (int dp = 0; dp < Lt::kPanels; ++dp)
+                        tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
+                               p.value_slab, policy);
+                }
+            } else {  // the block's own K / V (bf16): the operands read from the
+                      // stage; ring-slot operands are loaded by the conversion warps
+                mbar_arrive_expect_tx(full, (KF8 ? 0 : Lt::kTileBytes) +
+                                                (VF8 ? 0 : Lt::kTileBytes));
+#pragma unroll
+                for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                    if (!KF8) tma_4d(kdst + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
+                    if (!VF8) tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
+                }
+            }
+        }
+        __syncwarp();
+        if (ok) issued = j + 1;
+        walk_next(p, wl);
+        ++j;
+    };
+
     // every input (and the workspace) may be written by the previous kernel
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // the first loads of the speculative plan go out while the lengths are
+    // checked (no step here waits: fresh stages and query buffers only)
+    if (spec && warp == kProducerWarp)
+        while (j < ntiles && j < kStages && ok && !((j == 0 || wl.t == 0) && qseg + 1 >= 2))
+            produce();
     {
         const int P1 = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
         const int T1 = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
-        if (!(spec && __all_sync(kFull, P1 == sP && T1 == sT))) {
+        if (!(spec && __all_sync(kFull, P1 == sP && T1 == sT))) {  // the same in every warp
+            if (spec) {  // loads issued under the stale plan land, then the barriers restart
+                if (warp == kProducerWarp) {
+                    for (long long t = 0; t < issued; ++t)
+                        wait(b_full + 8 * (int)t, 0u, abort_flag, p.status);
+                    for (int q = 0; q <= qseg; ++q) wait(b_qfull + 8 * q, 0u, abort_flag, p.status);
+                }
+                __syncthreads();
+                if (threadIdx.x == 0) init_bars();
+                __syncthreads();
+            }
             lo = hi = 0;
             w0 = {0, 0, 0, 1, 0, 0};
             ntiles = plan(p, P1, T1, lo, hi, w0) ? hi - lo : 0;
+            wl = w0;
+            qseg = -1;
+            issued = j = 0;
+            ok = true;
         }
     }
 
@@ -760,72 +863,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         // Warp-uniform loop; one elected lane issues.  Stage s is reused once
         // the P V that read it has completed (the P V warp commits empty[s]);
         // a query buffer once the last S of the segment before last completed.
-        uint64_t policy;
-        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
-        Walk wl = w0;
-        int qseg = -1;
-        long long issued = 0;  // tiles whose loads were issued (and a query segment's)
-        bool ok = true;
-        for (long long j = 0; j < ntiles && ok; ++j) {
-            if (j == 0 || wl.t == 0) {  // the segment's query rows
-                ++qseg;
-                const int qb = qseg & 1;
-                if (qseg >= 2)
-                    ok = ok && wait(b_qempty + 8 * qb, (uint32_t)(((qseg - 2) >> 1) & 1),
-                                    abort_flag, p.status);
-                if (ok && elect_one()) {
-                    const uint32_t full = b_qfull + 8 * qb;
-                    const uint32_t dst = sbase + Lt::kQOff + qb * Lt::kQBytes;
-                    mbar_arrive_expect_tx(full, Lt::kPanels * p.rows_max * 128);
-#pragma unroll
-                    for (int dp = 0; dp < Lt::kPanels; ++dp)
-                        tma_4d(dst + dp * (kRows * 128), &tm_q, full, dp * 64, wl.h * p.G, 0,
-                               wl.b);
-                }
-            }
-            const int s = (int)(j % kStages);
-            if (j >= kStages)
-                ok = ok && wait(b_empty + 8 * s, (uint32_t)(((j - kStages) / kStages) & 1),
-                                abort_flag, p.status);
-            if (ok && elect_one()) {
-                const uint32_t full = b_full + 8 * s;
-                const uint32_t kdst = sbase + Lt::kStagesOff + s * Lt::kStageBytes;
-                const uint32_t vdst = kdst + Lt::kKBytes;
-                if (wl.t < wl.nt - 1) {
-                    const int tok = wl.t * kTileKeys;
-                    mbar_arrive_expect_tx(full, Lt::kStageBytes);
-                    // an e4m3 tile is one {D, 1, 64} box, a bf16 tile D / 64 swizzled panels
-                    if (KF8) {
-                        tma_5d(kdst, &tm_k, full, 0, wl.h, tok, wl.b, p.key_slab, policy);
-                    } else {
-#pragma unroll
-                        for (int dp = 0; dp < Lt::kPanels; ++dp)
-                            tma_5d(kdst + dp * 8192, &tm_k, full, dp * 64, wl.h, tok, wl.b,
-                                   p.key_slab, policy);
-                    }
-                    if (VF8) {
-                        tma_5d(vdst, &tm_v, full, 0, wl.h, tok, wl.b, p.value_slab, policy);
-                    } else {
-#pragma unroll
-                        for (int dp = 0; dp < Lt::kPanels; ++dp)
-                            tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
-                                   p.value_slab, policy);
-                    }
-                } else {  // the block's own K / V (bf16): the operands read from the
-                          // stage; ring-slot operands are loaded by the conversion warps
-                    mbar_arrive_expect_tx(full, (KF8 ? 0 : Lt::kTileBytes) +
-                                                    (VF8 ? 0 : Lt::kTileBytes));
-#pragma unroll
-                    for (int dp = 0; dp < Lt::kPanels; ++dp) {
-                        if (!KF8) tma_4d(kdst + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0, wl.b);
-                        if (!VF8) tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
-                    }
-                }
-            }
-            __syncwarp();
-            if (ok) issued = j + 1;
-            walk_next(p, wl);
-        }
+        while (j < ntiles && ok) produce();
         drain_tiles = issued;
         drain_qseg = qseg;
     } else if (warp == kMmaWarp || warp == kSWarp) {
