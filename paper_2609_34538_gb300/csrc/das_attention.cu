@@ -1102,19 +1102,28 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                     }
                 }
             }
-            // P = 2^(s - m) as bf16 into the swizzled P buffer (32 keys = 4 chunks)
+            // P = 2^(s - m) as bf16 into the swizzled P buffer (32 keys = 4
+            // chunks): all exponentials first, then the packs and a tree sum
+            // (measured faster than one loop that does all three per pair)
             const float mu = m_ref == -INFINITY ? 0.f : m_ref;
-            uint32_t w[16];
-            float l4[4] = {0.f, 0.f, 0.f, 0.f};
+            if (full_tile) {
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
-                const float a = full_tile ? ex2(fmaf(v[2 * e], scale, -mu)) : ex2(v[2 * e] - mu);
-                const float b2 =
-                    full_tile ? ex2(fmaf(v[2 * e + 1], scale, -mu)) : ex2(v[2 * e + 1] - mu);
-                l4[e & 3] += a + b2;
-                w[e] = pack_bf16(a, b2);
+                for (int j = 0; j < 32; ++j) v[j] = ex2(fmaf(v[j], scale, -mu));
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = ex2(v[j] - mu);
             }
-            const float lt = (l4[0] + l4[1]) + (l4[2] + l4[3]);
+            uint32_t w[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) w[e] = pack_bf16(v[2 * e], v[2 * e + 1]);
+            float t16[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) t16[j] = v[j] + v[j + 16];
+#pragma unroll
+            for (int wd = 8; wd > 0; wd >>= 1)
+#pragma unroll
+                for (int j = 0; j < wd; ++j) t16[j] += t16[j + wd];
+            const float lt = t16[0];
             // P buffer (k & 1) is free once P V of tile k-2, its last reader, is done
             // (pvdone[k & 1] completes once per P V of tiles with that parity)
             if (k >= 2) wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)(((k - 2) >> 1) & 1), abort_flag,
