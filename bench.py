@@ -51,7 +51,7 @@ def parse():
     ap.add_argument("--layers", type=int, default=0,
                     help="override the workload's layer count (smaller profiling captures)")
     ap.add_argument("--probe", default="",
-                    help="run only one probe (draft:long, draft:batched, e4m3:decode, "
+                    help="run only one probe (draft:long, draft:batched, draft:verify, e4m3:decode, "
                          "e4m3:long) with --steps/--warmup/--layers and print its result: "
                          "for profiling captures")
     ap.add_argument("--compact-depths", action="store_true",
@@ -308,7 +308,7 @@ def gpu_arm(args):
 
     probes = seq = wave = f8 = None
     if not args.no_probes:
-        probes = {n: draft_probe(n, dev, 200, 5, peak) for n in ("long", "batched")}
+        probes = {n: draft_probe(n, dev, 200, 5, peak) for n in ("long", "batched", "verify")}
         with torch.cuda.stream(stream):
             pl.copy_(P0)  # the timed steps committed onto the prefix
         seq = sequential_probe(wl, cache, pl, ws, dev, 20, 3, peak)
@@ -375,17 +375,21 @@ def gpu_arm(args):
 
 
 def draft_probe(name, dev, steps, warmup, peak, layers=0):
-    """Per-call time of another workload's draft phase, timed like the main
-    one (a CUDA graph of its L layer calls, L2 flushed before every replay).
-    Only the two depth slabs the calls read are stored (depths compacted to
-    key slab 1 and value slab 2): the bytes read are those of the full cache."""
+    """Per-call time of another workload's attention phase, timed like the
+    main one (a CUDA graph of its L layer calls, L2 flushed before every
+    replay).  Only the depth slabs the calls read are stored (a draft
+    workload's key and value depths compacted to slabs 1 and 2; a verify
+    workload's depth R, read for keys and values alike by
+    das_verify_attention, to slab 2): the bytes read are those of the full
+    cache."""
     import torch
 
     import paper_2609_34538_gb300 as das
     from synth import device as sdev
     from synth import workloads as wlm
 
-    wl = wlm.WORKLOADS[name].replace(depths=2, key_depth=1, value_depth=2)
+    verify = wlm.WORKLOADS[name].kind == "verify"
+    wl = wlm.WORKLOADS[name].replace(depths=2, key_depth=2 if verify else 1, value_depth=2)
     if layers:
         wl = wl.replace(layers=layers)
     L, B, W = wl.layers, wl.batch, wl.max_block
@@ -404,8 +408,12 @@ def draft_probe(name, dev, steps, warmup, peak, layers=0):
 
     def phase():
         for l, (q, kb, vb) in enumerate(ins):
-            das.das_mature_v_attention(cache, l, 1, 2, pl, bl, q, kb, vb, ws, out=outs[l][0],
-                                       lse=outs[l][1], stream=stream)
+            if verify:
+                das.das_verify_attention(cache, l, 2, pl, bl, q, kb, vb, ws, out=outs[l][0],
+                                         lse=outs[l][1], stream=stream)
+            else:
+                das.das_mature_v_attention(cache, l, 1, 2, pl, bl, q, kb, vb, ws,
+                                           out=outs[l][0], lse=outs[l][1], stream=stream)
 
     with torch.cuda.stream(stream):
         phase()
@@ -429,7 +437,9 @@ def draft_probe(name, dev, steps, warmup, peak, layers=0):
     gbs = nbytes * len(ms) / (sum(ms) / 1e3) / 1e9
     del K, V, cache, flush
     torch.cuda.empty_cache()
-    return {"workload": wl.name, "depth_slabs_stored": "2 (the key and value slabs read)",
+    return {"workload": wl.name,
+            "depth_slabs_stored": ("2 (depth R, read for keys and values)" if verify
+                                   else "2 (the key and value slabs read)"),
             "per_call_us": round(statistics.mean(ms) * 1e3 / L, 2), "gbs": round(gbs, 1),
             "pct_of_measured_hbm": round(100 * gbs / peak, 1),
             "pct_of_nominal_8000": round(100 * gbs / 8000.0, 1), "steps": len(ms)}

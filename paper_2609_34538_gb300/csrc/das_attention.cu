@@ -356,15 +356,15 @@ __device__ __forceinline__ void walk_next(const AttnParams &p, Walk &w) {
 }
 
 // Extra weight of a pair's block tile when the list is split.  Ending one
-// segment and starting the next (the mostly empty block tile holding a
-// pipeline slot, the partial write, the first tile's max pass) costs a CTA
-// more than one tile's time.  With few pairs per CTA (at least 4 CTAs per
-// pair) the CTAs whose range holds a block tile are a minority that finishes
-// last, so they take one tile fewer; with many pairs most ranges hold one
-// and the weight only moves work around (measured on the decode, long and
-// batched workloads).
-constexpr int kBlockWeight = 1;
-constexpr int kCtasPerPairForWeight = 4;
+// segment (the mostly empty block tile holding a pipeline slot, the wait for
+// the last P V, the partial write) costs a CTA about two tiles' time, so a
+// range that holds a block tile takes two tiles fewer while there is at
+// least one CTA per pair; with more pairs than CTAs nearly every range holds
+// one and the weight would only move work around (weights 1-3 and CTA-per-
+// pair thresholds 1 and 4 measured on the decode, long, batched and verify
+// workloads).
+constexpr int kBlockWeight = 2;
+constexpr int kCtasPerPairForWeight = 1;
 
 // The split of the tile list: tile x of pair q has weighted position
 // x + beta q; CTA c takes the tiles whose weighted position lies in
