@@ -1103,8 +1103,9 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 }
             }
             // P = 2^(s - m) as bf16 into the swizzled P buffer (32 keys = 4
-            // chunks): all exponentials first, then the packs and a tree sum
-            // (measured faster than one loop that does all three per pair)
+            // chunks): all exponentials first, then the packs (measured faster
+            // than one loop that does both per pair); their tree sum for l
+            // comes after P has been handed on
             const float mu = m_ref == -INFINITY ? 0.f : m_ref;
             if (full_tile) {
 #pragma unroll
@@ -1116,14 +1117,6 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             uint32_t w[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) w[e] = pack_bf16(v[2 * e], v[2 * e + 1]);
-            float t16[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) t16[j] = v[j] + v[j + 16];
-#pragma unroll
-            for (int wd = 8; wd > 0; wd >>= 1)
-#pragma unroll
-                for (int j = 0; j < wd; ++j) t16[j] += t16[j + wd];
-            const float lt = t16[0];
             // P buffer (k & 1) is free once P V of tile k-2, its last reader, is done
             // (pvdone[k & 1] completes once per P V of tiles with that parity)
             if (k >= 2) wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)(((k - 2) >> 1) & 1), abort_flag,
@@ -1137,7 +1130,6 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                              "r"(w[4 * q4]), "r"(w[4 * q4 + 1]), "r"(w[4 * q4 + 2]),
                              "r"(w[4 * q4 + 3])
                              : "memory");
-            l_sum += lt;
             // keys past the end of the tile may hold anything: zero their V rows
             if (nvalid < kTileKeys) {
                 const uint32_t vt = v_src(s, k);
@@ -1156,6 +1148,16 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
+            {  // the row sum is needed only for l: after P has been handed on
+                float t16[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) t16[j] = v[j] + v[j + 16];
+#pragma unroll
+                for (int wd = 8; wd > 0; wd >>= 1)
+#pragma unroll
+                    for (int j = 0; j < wd; ++j) t16[j] += t16[j + wd];
+                l_sum += t16[0];
+            }
 
             // ---- end of segment: O / l and lse ----
             if (last) {
