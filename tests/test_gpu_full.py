@@ -101,3 +101,50 @@ def test_full_size_accept_and_append():
     finally:
         del cache, K, V, kn, vn
         torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("name", ["decode", "long"])
+def test_full_size_sampled_e4m3(name):
+    """The e4m3 cache variant at full size, configured as the benchmark's
+    e4m3 probe: keys at depth r = 1 stored as e4m3 codes (host generator),
+    values at depth R = 2 as bf16 (device fill, checked bit for bit against
+    the host generator on the sampled slabs).  Sampled (sequence, kv head)
+    groups are recomputed by the oracle from the widened keys; every output
+    is checked for the properties that hold at any size."""
+    import paper_2609_34538_gb300 as das
+    wl = wl_mod.WORKLOADS[name].replace(depths=2, key_depth=1, value_depth=2)
+    L, B, cap, H, D, G = wl.layers, wl.batch, wl.capacity, wl.kv_heads, wl.head_dim, wl.group
+    cache = das.DepthKVCacheF8.empty(2, L, B, cap, H, D)
+    codes = synth.e4m3_codes(wl.seed, synth.T_KLOW, (1, L, B, cap, H, D))
+    cache.k_low.copy_(torch.from_numpy(codes))
+    sdev.fill_matured(cache.v_top, wl.seed, synth.T_VCACHE, 1, 2, 2)
+    ws = das.new_workspace_f8(cache, wl.q_heads, wl.max_block)
+    P, T = wl.prefix_lens(), wl.block_lens()
+    pl, bl = dev_i32(P), dev_i32(T)
+    try:
+        for layer in range(L):
+            q, kb, vb = sdev.layer_inputs(wl, layer)
+            out, lse = das.das_mature_v_attention_f8(cache, layer, 1, 2, pl, bl, q, kb, vb, ws)
+            torch.cuda.synchronize()
+            o = out.float().cpu().numpy()
+            l = lse.cpu().numpy()
+            assert np.all(np.isfinite(o))
+            for b in range(B):
+                assert np.all(o[b, T[b]:] == 0) and np.all(np.isneginf(l[b, :, T[b]:]))
+                assert np.all(np.isfinite(l[b, :, :T[b]]))
+            qh, kbh, vbh = host_bits(q), host_bits(kb), host_bits(vb)
+            for b, h in _pairs(wl, layer, 2 if wl.max_prefix > 20000 else 3):
+                kc = codes[0, layer, b, :P[b], h:h + 1]
+                kp = oracle.widen_f8_cache(np.zeros(kc.shape, np.uint16), kc[None])[0]
+                vp = synth.matured_block(wl.seed, synth.T_VCACHE, 1, 2, 2, layer, b, 0, int(P[b]),
+                                         h, h + 1, D)
+                assert np.array_equal(host_bits(cache.v_top[layer, b, :P[b], h:h + 1]), vp)
+                ro, rl = oracle.attend_seq(qh[b, :, h * G:(h + 1) * G], kp, vp,
+                                           kbh[b, :, h:h + 1], vbh[b, :, h:h + 1],
+                                           block_len=int(T[b]))
+                assert_close(o[b, :, h * G:(h + 1) * G], ro, l[b, h * G:(h + 1) * G], rl,
+                             where=f"[{name} e4m3 keys, layer {layer} b {b} kv head {h}]")
+        assert das.workspace_status(ws) == 0
+    finally:
+        del cache
+        torch.cuda.empty_cache()
