@@ -5,6 +5,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 from synth import workloads as wl_mod
 from tests.gpu_util import assert_close, dev_bf16, dev_i32, run_small
 
@@ -129,6 +130,10 @@ def test_out_of_range_lengths_are_clamped_and_flagged():
     torch.cuda.synchronize()
     assert das.workspace_status(ws) == 2 and das.workspace_status(ws2) == 0
     assert torch.equal(out1, out2) and torch.equal(l1, l2)
+    # a prefix that fills the whole capacity, against the oracle
+    ro, rl = oracle.attention(K, V, 0, 2, 8, np.array([cap], np.int32), np.array([4], np.int32),
+                              wl_mod.gen_q(wl, 0), *wl_mod.gen_block_kv(wl, 0))
+    assert_close(out2.float().cpu().numpy(), ro, l2.cpu().numpy(), rl, where="[P = capacity]")
 
 
 def test_deterministic_and_graph_capturable():
