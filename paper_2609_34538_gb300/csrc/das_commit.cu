@@ -4,6 +4,8 @@
 // Every kernel here is launched as a programmatic dependent of the previous
 // kernel in the stream: it reads nothing before griddepcontrol.wait, and
 // every CTA executes that wait.
+#include <atomic>
+
 #include <cooperative_groups.h>
 
 #include "das_internal.h"
@@ -14,20 +16,23 @@ namespace das {
 namespace {
 
 // ---- greedy acceptance and the DAS-Wave readout ------------------------------
-// One cluster of kAcceptCtas CTAs per sequence.  CTA j of the cluster scans
-// slice j of the vocabulary for every row i < W of its sequence and keeps its
-// best (value, index) per row in shared memory; after a cluster barrier CTA 0
-// reads the kAcceptCtas candidates of each row through distributed shared
-// memory and
+// One cluster of CTAS CTAs per sequence (CTAS = 16 for up to four sequences,
+// which spreads a sequence's logits over more SMs, else 8: with more
+// sequences, 16-CTA clusters measured slower than 8-CTA ones).  CTA r of the
+// cluster scans slice r of the vocabulary for every row i < W of its sequence
+// and stores its best (value, index) per row straight into CTA 0's shared
+// memory (distributed shared memory).  The others then arrive at the cluster
+// barrier and exit; CTA 0 waits for them, reduces the CTAS candidates of each
+// row from its own shared memory and
 //   - accept mode (Sec. 3.4): writes target_ids, counts the accepted prefix
 //     and writes accepted and next_token;
 //   - readout mode (Eq. 6, Sec. 3.3): writes the argmax of row i as the guess
 //     of position i + 1, tokens[b][i + 1].
-constexpr int kAcceptCtas = 8;
 constexpr int kAcceptThreads = 1024;
 constexpr int kAcceptWarps = kAcceptThreads / 32;
 constexpr int kMaxW = 1024;
-constexpr int kBatch = 8;  // vector loads in flight per thread
+constexpr int kBatch = 8;          // vector loads in flight per thread
+constexpr int kWideClusterMaxB = 4;  // sequences up to which a cluster has 16 CTAs
 
 // (value, index) order of the argmax: larger value wins, equal values go to
 // the smaller index, so the result is the first maximum.
@@ -46,14 +51,11 @@ __device__ __forceinline__ void warp_best(float &bv, int &bi) {
     }
 }
 
-struct AcceptSmem {
-    float cand_v[kMaxW];  // this CTA's best per row
-    int cand_i[kMaxW];
-    float warp_v[kAcceptWarps];
-    int warp_i[kAcceptWarps];
-    int target[kMaxW];  // CTA 0: the row argmaxes
-    int first_miss;
-};
+// dynamic shared memory of an accept CTA: candidate values [CTAS][W] and
+// indices [CTAS][W] (filled in CTA 0 by every CTA), row argmaxes [W] (CTA 0)
+__host__ __device__ constexpr size_t accept_smem_bytes(int ctas, int W) {
+    return (size_t)ctas * W * 8 + (size_t)W * 4;
+}
 
 struct ArgmaxArgs {
     const float *logits;  // [B][W][vocab]
@@ -67,17 +69,28 @@ struct ArgmaxArgs {
 };
 
 // VEC = 4: float4 loads (vocab % 4 == 0 and 16-byte aligned logits), else 1.
-template <int VEC, bool READOUT>
+template <int VEC, bool READOUT, int CTAS>
 __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const ArgmaxArgs a) {
     const float *__restrict__ logits = a.logits;
     const int W = a.W, vocab = a.vocab, slice = a.slice;
-    __shared__ AcceptSmem sm;
+    extern __shared__ __align__(16) uint8_t accept_smem[];
+    float *cand_v = reinterpret_cast<float *>(accept_smem);
+    int *cand_i = reinterpret_cast<int *>(cand_v + CTAS * W);
+    int *target = cand_i + CTAS * W;
+    __shared__ float warp_v[kAcceptWarps];
+    __shared__ int warp_i[kAcceptWarps];
+    __shared__ int first_miss;
     cg::cluster_group cluster = cg::this_cluster();
     const int rank = (int)cluster.block_rank();
-    const int b = blockIdx.x / kAcceptCtas;
+    const int b = blockIdx.x / CTAS;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // a CTA's shared memory may be written by another only once that CTA has
+    // started: every CTA arrives here and waits before its first remote store
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    float *dst_v = cluster.map_shared_rank(cand_v, 0) + rank * W;
+    int *dst_i = cluster.map_shared_rank(cand_i, 0) + rank * W;
 
     // threads per row: the CTA's warps split over min(W, 32) rows at a time
     int tpr = kAcceptThreads;
@@ -94,19 +107,19 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const ArgmaxArgs
             const float *row = logits + ((size_t)b * W + i) * (size_t)vocab + lo;
             // batches of kBatch vector loads, all issued before the compares
             for (int j0 = part; j0 < nvec; j0 += kBatch * tpr) {
-                float a[kBatch][VEC];
+                float x[kBatch][VEC];
 #pragma unroll
                 for (int u = 0; u < kBatch; ++u) {
                     const int j = j0 + u * tpr;
                     if (j < nvec) {
                         if (VEC == 4) {
-                            const float4 x = __ldcs(reinterpret_cast<const float4 *>(row) + j);
-                            a[u][0] = x.x;
-                            a[u][1 % VEC] = x.y;
-                            a[u][2 % VEC] = x.z;
-                            a[u][VEC - 1] = x.w;
+                            const float4 y = __ldcs(reinterpret_cast<const float4 *>(row) + j);
+                            x[u][0] = y.x;
+                            x[u][1 % VEC] = y.y;
+                            x[u][2 % VEC] = y.z;
+                            x[u][VEC - 1] = y.w;
                         } else {
-                            a[u][0] = __ldcs(row + j);
+                            x[u][0] = __ldcs(row + j);
                         }
                     }
                 }
@@ -115,61 +128,60 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const ArgmaxArgs
                     const int j = j0 + u * tpr;
                     if (j < nvec) {
 #pragma unroll
-                        for (int e = 0; e < VEC; ++e) better(bv, bi, a[u][e], lo + VEC * j + e);
+                        for (int e = 0; e < VEC; ++e) better(bv, bi, x[u][e], lo + VEC * j + e);
                     }
                 }
             }
         }
         warp_best(bv, bi);
         if (lane == 0) {
-            sm.warp_v[warp] = bv;
-            sm.warp_i[warp] = bi;
+            warp_v[warp] = bv;
+            warp_i[warp] = bi;
         }
         __syncthreads();
+        if (i0 == 0) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
         if (threadIdx.x < rows_per_pass && i0 + (int)threadIdx.x < W) {
             float v = -INFINITY;
-            int x = 0x7fffffff;
+            int y = 0x7fffffff;
             for (int w = 0; w < warps_per_row; ++w)
-                better(v, x, sm.warp_v[threadIdx.x * warps_per_row + w],
-                       sm.warp_i[threadIdx.x * warps_per_row + w]);
-            sm.cand_v[i0 + threadIdx.x] = v;
-            sm.cand_i[i0 + threadIdx.x] = x;
+                better(v, y, warp_v[threadIdx.x * warps_per_row + w],
+                       warp_i[threadIdx.x * warps_per_row + w]);
+            dst_v[i0 + threadIdx.x] = v;
+            dst_i[i0 + threadIdx.x] = y;
         }
         __syncthreads();
     }
-    cluster.sync();  // every CTA's candidates are in its shared memory
+    // the candidates are in CTA 0 once every CTA has arrived (release); only
+    // CTA 0 waits, and no CTA's shared memory but CTA 0's is ever read remotely
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    if (rank != 0) return;
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 
-    if (rank == 0) {
-        if (threadIdx.x == 0) sm.first_miss = W;
-        __syncthreads();
-        for (int i = threadIdx.x; i < W; i += kAcceptThreads) {
-            float v = -INFINITY;
-            int x = 0x7fffffff;
+    if (threadIdx.x == 0) first_miss = W;
+    __syncthreads();
+    for (int i = threadIdx.x; i < W; i += kAcceptThreads) {
+        float v = -INFINITY;
+        int x = 0x7fffffff;
 #pragma unroll
-            for (int r = 0; r < kAcceptCtas; ++r) {
-                const AcceptSmem *o = cluster.map_shared_rank(&sm, r);
-                better(v, x, o->cand_v[i], o->cand_i[i]);
-            }
-            // a row of -inf keeps the sentinel: the first index wins
-            const int t = x == 0x7fffffff ? 0 : x;
-            if (READOUT) {
-                a.tokens[(size_t)b * a.stride + i + 1] = t;
-            } else {
-                sm.target[i] = t;
-                a.target_ids[(size_t)b * W + i] = t;
-                if (a.draft[(size_t)b * W + i] != t) atomicMin(&sm.first_miss, i);
-            }
-        }
-        if (!READOUT) {
-            __syncthreads();
-            if (threadIdx.x == 0) {
-                const int n = sm.first_miss;
-                a.accepted[b] = n;
-                a.next_token[b] = n < W ? sm.target[n] : a.draft[(size_t)b * W + W - 1];
-            }
+        for (int r = 0; r < CTAS; ++r) better(v, x, cand_v[r * W + i], cand_i[r * W + i]);
+        // a row of -inf keeps the sentinel: the first index wins
+        const int t = x == 0x7fffffff ? 0 : x;
+        if (READOUT) {
+            a.tokens[(size_t)b * a.stride + i + 1] = t;
+        } else {
+            target[i] = t;
+            a.target_ids[(size_t)b * W + i] = t;
+            if (a.draft[(size_t)b * W + i] != t) atomicMin(&first_miss, i);
         }
     }
-    cluster.sync();  // CTA 0 has read the others' shared memory
+    if (!READOUT) {
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int n = first_miss;
+            a.accepted[b] = n;
+            a.next_token[b] = n < W ? target[n] : a.draft[(size_t)b * W + W - 1];
+        }
+    }
 }
 
 // ---- commit ---------------------------------------------------------------------
@@ -336,20 +348,96 @@ cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, unsigne
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
 }
 
-cudaError_t argmax_launch(const ArgmaxArgs &a0, int B, bool readout, cudaStream_t stream) {
-    if (B == 0) return cudaSuccess;
-    if (a0.W > kMaxW || B > 0x7fffffff / kAcceptCtas) return cudaErrorInvalidValue;
-    ArgmaxArgs a = a0;
-    const bool vec = (a.vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(a.logits) & 15u) == 0;
+// The dynamic shared memory opt-in (and, for 16-CTA clusters, the non-portable
+// cluster size) of one accept kernel, once per device.  Returns false if the
+// kernel cannot run with that many CTAs per cluster on this device.
+template <int VEC, bool READOUT, int CTAS>
+cudaError_t accept_configure(int dev, bool &usable) {
+    static std::atomic<int> state[64];  // 0 unknown, 1 usable, 2 not usable
+    usable = false;
+    if (dev < 64) {
+        const int st = state[dev].load(std::memory_order_acquire);
+        if (st != 0) {
+            usable = st == 1;
+            return cudaSuccess;
+        }
+    }
+    auto kernel = accept_kernel<VEC, READOUT, CTAS>;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)accept_smem_bytes(CTAS, kMaxW));
+    if (e != cudaSuccess) return e;
+    if (CTAS > 8) {
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(CTAS);
+        cfg.blockDim = dim3(kAcceptThreads);
+        cfg.dynamicSmemBytes = accept_smem_bytes(CTAS, kMaxW);
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = CTAS;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int clusters = 0;
+        e = cudaOccupancyMaxActiveClusters(&clusters, kernel, &cfg);
+        if (e != cudaSuccess) return e;
+        usable = clusters >= 1;
+    } else {
+        usable = true;
+    }
+    if (dev < 64) state[dev].store(usable ? 1 : 2, std::memory_order_release);
+    return cudaSuccess;
+}
+
+template <int VEC, bool READOUT, int CTAS>
+cudaError_t argmax_launch_ctas(ArgmaxArgs a, int B, cudaStream_t stream) {
     // slices are whole float4s
-    int slice = (a.vocab + kAcceptCtas - 1) / kAcceptCtas;
+    const int slice = (a.vocab + CTAS - 1) / CTAS;
     a.slice = (slice + 3) & ~3;
-    const dim3 grid((unsigned)(B * kAcceptCtas)), block(kAcceptThreads);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(B * CTAS));
+    cfg.blockDim = dim3(kAcceptThreads);
+    cfg.dynamicSmemBytes = accept_smem_bytes(CTAS, a.W);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = CTAS;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, accept_kernel<VEC, READOUT, CTAS>, a);
+}
+
+template <int VEC, bool READOUT>
+cudaError_t argmax_launch_vec(const ArgmaxArgs &a, int B, cudaStream_t stream) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    bool usable = false;
+    if (B <= kWideClusterMaxB) {
+        e = accept_configure<VEC, READOUT, 16>(dev, usable);
+        if (e != cudaSuccess) return e;
+        if (usable) return argmax_launch_ctas<VEC, READOUT, 16>(a, B, stream);
+    }
+    e = accept_configure<VEC, READOUT, 8>(dev, usable);
+    if (e != cudaSuccess) return e;
+    return argmax_launch_ctas<VEC, READOUT, 8>(a, B, stream);
+}
+
+cudaError_t argmax_launch(const ArgmaxArgs &a, int B, bool readout, cudaStream_t stream) {
+    if (B == 0) return cudaSuccess;
+    if (a.W < 1 || a.W > kMaxW || B > 0x7fffffff / 16) return cudaErrorInvalidValue;
+    const bool vec = (a.vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(a.logits) & 15u) == 0;
     if (readout)
-        return vec ? launch_pdl(accept_kernel<4, true>, grid, block, kAcceptCtas, stream, a)
-                   : launch_pdl(accept_kernel<1, true>, grid, block, kAcceptCtas, stream, a);
-    return vec ? launch_pdl(accept_kernel<4, false>, grid, block, kAcceptCtas, stream, a)
-               : launch_pdl(accept_kernel<1, false>, grid, block, kAcceptCtas, stream, a);
+        return vec ? argmax_launch_vec<4, true>(a, B, stream)
+                   : argmax_launch_vec<1, true>(a, B, stream);
+    return vec ? argmax_launch_vec<4, false>(a, B, stream)
+               : argmax_launch_vec<1, false>(a, B, stream);
 }
 
 }  // namespace

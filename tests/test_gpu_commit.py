@@ -56,6 +56,23 @@ def test_accept_ties_and_infinities():
     assert list(acc) == [4, 3, 3]
 
 
+@pytest.mark.parametrize("B", [1, 8])
+def test_accept_ties_across_slices(B):
+    """Equal maxima in two CTAs' vocabulary slices: a sequence is scanned by
+    16 CTAs (slices of 260 columns at V = 4099) for up to four sequences and
+    by 8 (slices of 516) beyond; the smaller index wins either way."""
+    W, V = 3, 4099
+    logits = np.zeros((B, W, V), dtype=np.float32)
+    logits[:, 0, [259, 260]] = 5.0
+    logits[:, 1, [515, 516]] = 5.0
+    logits[:, 2, [V - 1, 0]] = 5.0
+    draft = np.zeros((B, W), dtype=np.int32)
+    draft[:, 0], draft[:, 1] = 259, 515
+    acc, tid, _ = check_accept(logits, draft)
+    assert np.all(tid[:, 0] == 259) and np.all(tid[:, 1] == 515) and np.all(tid[:, 2] == 0)
+    assert np.all(acc == 3)
+
+
 def _append_case(R, L, B, cap, H, D, W, pl, acc, seed):
     import paper_2609_34538_gb300 as das
     rng = np.random.default_rng(seed)
