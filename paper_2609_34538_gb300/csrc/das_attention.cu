@@ -44,6 +44,7 @@
 // freed before the CTA exits.
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <atomic>
 
 #include "das_internal.h"
@@ -1256,14 +1257,17 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
 // and rows past the block get 0 and lse -inf.  The pair's segments are found
 // from the lengths before griddepcontrol.wait (the attention grid this one
 // depends on started after every kernel that could write them had
-// completed); the partials are read after it, 8 segments' loads in flight.
+// completed); the partials are read after it, SEGS segments' loads in
+// flight.  SEGS trades round trips for registers: at D = 128, 8 segments take
+// 116 registers a thread (4 CTAs per SM), 4 take 72 (7), 2 take 40 (12).
 constexpr int kMergeWarps = 4;
 
-template <int D>
-__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParams p) {
+template <int D, int SEGS>
+__global__ void __launch_bounds__(kMergeWarps * 32, SEGS == 2 ? 12 : SEGS == 4 ? 7 : 4)
+    merge_kernel(const AttnParams p) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     constexpr int VPL = D / 32;
-    constexpr int kSegs = 8;
+    constexpr int kSegs = SEGS;
     const int rblocks = (p.rows_max + kMergeWarps - 1) / kMergeWarps;
     const int pair = blockIdx.x / rblocks;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1360,6 +1364,33 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const AttnParam
     if (lane == 0) *lrow = L > 0.f ? M + __logf(L) : -INFINITY;
 }
 
+// Resident merge CTAs per SM for the 8-, 4- and 2-segment variants, looked
+// up once per device.
+template <int D>
+cudaError_t merge_occupancy(int dev, int occ[3]) {
+    static std::atomic<int> cached[64][3];
+    if (dev < 64 && cached[dev][2].load(std::memory_order_acquire) > 0) {
+        for (int v = 0; v < 3; ++v) occ[v] = cached[dev][v].load(std::memory_order_relaxed);
+        return cudaSuccess;
+    }
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[0], merge_kernel<D, 8>,
+                                                                  kMergeWarps * 32, 0);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[1], merge_kernel<D, 4>,
+                                                          kMergeWarps * 32, 0);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[2], merge_kernel<D, 2>,
+                                                          kMergeWarps * 32, 0);
+    if (e != cudaSuccess) return e;
+    for (int v = 0; v < 3; ++v) occ[v] = std::max(occ[v], 1);
+    if (dev < 64) {
+        cached[dev][0].store(occ[0], std::memory_order_relaxed);
+        cached[dev][1].store(occ[1], std::memory_order_relaxed);
+        cached[dev][2].store(occ[2], std::memory_order_release);
+    }
+    return cudaSuccess;
+}
+
 template <int D, bool KF8, bool VF8>
 cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
                      const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
@@ -1388,11 +1419,31 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8>, tk, tv, tkb, tvb, tq, p);
     if (e != cudaSuccess) return e;
-    cfg.gridDim = dim3((unsigned)((long long)p.B * p.Hkv *
-                                  ((p.rows_max + kMergeWarps - 1) / kMergeWarps)));
+    const long long ctas = (long long)p.B * p.Hkv * ((p.rows_max + kMergeWarps - 1) / kMergeWarps);
+    cfg.gridDim = dim3((unsigned)ctas);
     cfg.blockDim = dim3(kMergeWarps * 32);
     cfg.dynamicSmemBytes = 0;
-    return cudaLaunchKernelEx(&cfg, merge_kernel<D>, p);
+    // The merge variant with the fewest estimated sequential steps: waves of
+    // resident merge CTAs (at least one) times L2 round trips per row (at
+    // least one), for a pair's average segment count 1 + C / (B Hkv).
+    const double segs = 1.0 + (double)p.num_ctas / ((double)p.B * p.Hkv);
+    int occ[3];
+    e = merge_occupancy<D>(dev, occ);
+    if (e != cudaSuccess) return e;
+    const int seg_of[3] = {8, 4, 2};
+    int best = 0;
+    double best_cost = 0.0;
+    for (int v = 0; v < 3; ++v) {
+        const double waves = std::max(1.0, (double)ctas / ((double)occ[v] * p.num_ctas));
+        const double cost = waves * std::max(1.0, segs / seg_of[v]);
+        if (v == 0 || cost < best_cost) {
+            best = v;
+            best_cost = cost;
+        }
+    }
+    if (best == 0) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 8>, p);
+    if (best == 1) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 4>, p);
+    return cudaLaunchKernelEx(&cfg, merge_kernel<D, 2>, p);
 }
 
 }  // namespace tc
