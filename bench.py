@@ -103,11 +103,42 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def code_digest(path):
+    """code_text_digest of a source file."""
+    return code_text_digest(open(path, encoding="utf-8").read())
+
+
+def code_text_digest(text):
+    """First 16 hex digits of the sha256 of a C/C++/CUDA source with its
+    comments, trailing blanks and empty lines removed (string and character
+    literals kept), so that an edit of comments alone keeps the digest."""
+    out, i, n = [], 0, len(text)
+    while i < n:
+        c = text[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and text[j] != c:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        elif text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    code = "\n".join(line.rstrip() for line in "".join(out).splitlines() if line.strip())
+    return hashlib.sha256(code.encode()).hexdigest()[:16]
+
+
 def kernel_traffic(workload):
     """dram bytes per attention launch from the committed ncu summary, if the
-    kernel source has not changed since it was captured; else None."""
+    kernel's code has not changed since it was captured; else None."""
     src = os.path.join(ROOT, "paper_2609_34538_gb300", "csrc", "das_attention.cu")
-    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    digest = code_digest(src)
     path = os.path.join(ROOT, "profiles", "attn_kernel_traffic.txt")
     if not os.path.exists(path):
         return None

@@ -4,12 +4,14 @@
 //
 // Work decomposition: every (sequence, kv head) pair owns ceil(P/64) prefix
 // tiles plus one block tile; all pairs' tiles form one list of N tiles, and
-// CTA c of a persistent grid of C CTAs (one per SM) takes the range
-// [c N / C, (c+1) N / C), cut into segments at pair boundaries.  A segment
-// that covers its pair writes the output.  The others write a partial (O / l
-// and the log-sum-exp of their keys) to the workspace, and merge_kernel,
-// launched right after as a programmatic dependent, combines each split
-// pair's partials by log-sum-exp.
+// CTA c of a persistent grid of C CTAs (one per SM) takes the c-th of C
+// equal ranges of that list (block tiles weighted for their extra cost, see
+// kBlockWeight), cut into segments at pair boundaries.  A segment that covers
+// its pair writes the output.  The others write a partial (O / l and the
+// log-sum-exp of their keys) to the workspace, and merge_kernel, launched
+// right after as a programmatic dependent, combines each split pair's
+// partials by log-sum-exp (8, 4 or 2 segments' loads in flight, chosen per
+// launch).
 //
 // One CTA = four softmax warps + one TMA warp + two MMA warps (+ four
 // conversion warps when prefix keys or values are stored as e4m3).
