@@ -214,12 +214,16 @@ das_status das_kv_append(const das_kv_cache *cache, const void *k_new, const voi
  *     DAS_NOALLOC_SCRATCH_BYTES (das_workspace_size() tells how much), with
  *     nothing launched.
  *   - The first call on a device looks up the array's device address (set-up
- *     done once per device); make that first call before any CUDA graph
- *     capture on that device.
+ *     done once per device, then kept); make that first call before any CUDA
+ *     graph capture on that device.  After cudaDeviceReset on a device, later
+ *     calls in that process are invalid.
  *   - All calls share the array and it keeps the last call's contents: calls
  *     that overlap in time on the GPU race and must be ordered by the caller.
- *     Each call clears the status word at the array's head; the bits of a
- *     call's device-side checks can be read there until the next call.
+ *     A call that passes its argument checks clears the status word at the
+ *     array's head (on `stream`, just before its kernels); its bits, as for
+ *     the workspace status word of das_mature_v_attention, are read with
+ *     das_noalloc_status until the next call.  A call that returns an error
+ *     enqueues nothing.
  */
 das_status das_mature_v_attention_noalloc(const das_kv_cache *cache, int layer, int key_depth,
                                           int value_depth, const int32_t *prefix_len,
@@ -227,6 +231,15 @@ das_status das_mature_v_attention_noalloc(const das_kv_cache *cache, int layer, 
                                           const void *k_blk, const void *v_blk, int num_q_heads,
                                           float softmax_scale, void *out, float *lse,
                                           void *stream);
+
+/*
+ * Copies the status word of das_mature_v_attention_noalloc's scratch on the
+ * current device (bit 0: an internal wait timed out; bit 1: a prefix or block
+ * length was out of range and clamped) to `dst` (host or device memory,
+ * 4 bytes) on `stream`, after the work enqueued there before it.  Allocates
+ * nothing.  The paper has no counterpart.
+ */
+das_status das_noalloc_status(int32_t *dst, void *stream);
 
 /*
  * A depth-indexed cache whose depths below R are stored as 8-bit floats.

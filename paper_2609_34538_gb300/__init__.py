@@ -81,6 +81,8 @@ def _load():
     lib.das_kv_append_f8.restype = i
     lib.das_mature_v_attention_noalloc.argtypes = [cp, i, i, i, p, p, i, p, p, p, i, f, p, p, p]
     lib.das_mature_v_attention_noalloc.restype = i
+    lib.das_noalloc_status.argtypes = [p, p]
+    lib.das_noalloc_status.restype = i
     lib.das_status_string.argtypes = [i]
     lib.das_status_string.restype = ctypes.c_char_p
     return lib
@@ -161,7 +163,10 @@ def workspace_status(workspace):
     return int(workspace[:4].view(torch.int32).item())
 
 
-def _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse, workspace):
+def _attention_shapes(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse):
+    """Checks every tensor of an attention call against the cache's shape
+    (allocating out / lse when omitted); returns (max_block, Hq, out, lse).
+    Raises before anything is launched."""
     _need(prefix_len, torch.int32, "prefix_len", 1)
     _need(block_len, torch.int32, "block_len", 1)
     _need(q, torch.bfloat16, "q", 4)
@@ -181,6 +186,11 @@ def _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse, wor
     _need(lse, torch.float32, "lse", 3)
     if tuple(out.shape) != tuple(q.shape) or tuple(lse.shape) != (B, Hq, T):
         raise ValueError("out must be like q and lse [batch][num_q_heads][max_block]")
+    return T, Hq, out, lse
+
+
+def _attention_args(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse, workspace):
+    T, Hq, out, lse = _attention_shapes(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse)
     _need(workspace, torch.uint8, "workspace", 1)
     return T, Hq, out, lse
 
@@ -205,23 +215,24 @@ def das_mature_v_attention_noalloc(cache, layer, key_depth, value_depth, prefix_
     the split-K scratch is a fixed array inside the library (shared by every
     call on a device; calls that overlap on the GPU race).  `out` and `lse`
     must be given by such callers; they are allocated here only for
-    convenience when omitted."""
-    R, L, B, cap, H, D = cache.shape
-    T, Hq = q.shape[1], q.shape[2]
-    if out is None:
-        out = torch.empty_like(q)
-    if lse is None:
-        lse = torch.empty((B, Hq, T), dtype=torch.float32, device=q.device)
-    _need(prefix_len, torch.int32, "prefix_len", 1)
-    _need(block_len, torch.int32, "block_len", 1)
-    for t, n in ((q, "q"), (k_blk, "k_blk"), (v_blk, "v_blk"), (out, "out")):
-        _need(t, torch.bfloat16, n, 4)
-    _need(lse, torch.float32, "lse", 3)
+    convenience when omitted.  Shapes are checked as for the workspace entry
+    point, before anything is launched."""
+    T, Hq, out, lse = _attention_shapes(cache, prefix_len, block_len, q, k_blk, v_blk, out, lse)
     _check(LIB.das_mature_v_attention_noalloc(
         ctypes.byref(cache.desc), layer, key_depth, value_depth, _ptr(prefix_len),
         _ptr(block_len), T, _ptr(q), _ptr(k_blk), _ptr(v_blk), Hq, float(softmax_scale),
         _ptr(out), _ptr(lse), _stream(stream)), "das_mature_v_attention_noalloc")
     return out, lse
+
+
+def noalloc_status(stream=None):
+    """The status word of the last das_mature_v_attention_noalloc call on the
+    current device (bits as workspace_status).  Synchronises the stream."""
+    host = torch.zeros(1, dtype=torch.int32)
+    s = torch.cuda.current_stream() if stream is None else stream
+    _check(LIB.das_noalloc_status(host.data_ptr(), s.cuda_stream), "das_noalloc_status")
+    s.synchronize()
+    return int(host.item())
 
 
 def das_verify_attention(cache, layer, depth, prefix_len, block_len, q, k_blk, v_blk, workspace,

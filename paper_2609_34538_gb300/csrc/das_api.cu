@@ -160,7 +160,7 @@ das_status attention_core(const Shape &c, int layer, Operand key, Operand value,
                           const int32_t *prefix_len, const int32_t *block_len, int max_block,
                           const void *q, const void *k_blk, const void *v_blk, int num_q_heads,
                           float softmax_scale, void *out, float *lse, void *workspace,
-                          size_t workspace_bytes, void *stream) {
+                          size_t workspace_bytes, bool clear_status, void *stream) {
     if (layer < 0 || layer >= c.layers || !prefix_len || !block_len || !q || !k_blk || !v_blk ||
         !out || !lse || num_q_heads < 1 || max_block < 1 || num_q_heads % c.kv_heads != 0 ||
         !aligned16(q) || !aligned16(k_blk) || !aligned16(v_blk) || !aligned16(out) ||
@@ -219,16 +219,22 @@ das_status attention_core(const Shape &c, int layer, Operand key, Operand value,
     p.scale_log2 = (float)(scale * 1.4426950408889634);
     p.num_ctas = attn_grid_size(dev);
     attn_workspace_layout(workspace, c.batch, c.kv_heads, p.rows_max, D, p.num_ctas, p);
+    // every argument is valid from here on: the only work before the launch
+    if (clear_status && cudaMemsetAsync(workspace, 0, kWorkspaceHeader,
+                                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return DAS_ERR_CUDA;
     const cudaError_t e = attn_launch(p, D, key.e4m3, value.e4m3, tk, tv, tkb, tvb, tq,
                                       static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? DAS_OK : DAS_ERR_CUDA;
 }
 
+}  // namespace
+
 das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_depth,
                      const int32_t *prefix_len, const int32_t *block_len, int max_block,
                      const void *q, const void *k_blk, const void *v_blk, int num_q_heads,
                      float softmax_scale, void *out, float *lse, void *workspace,
-                     size_t workspace_bytes, void *stream) {
+                     size_t workspace_bytes, bool clear_status, void *stream) {
     if (!cache_ok(c)) {
         if (c && c->head_dim != 64 && c->head_dim != 128 && c->k && c->v) return DAS_ERR_UNSUPPORTED;
         return DAS_ERR_INVALID_ARG;
@@ -240,8 +246,10 @@ das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_
     return attention_core(sh, layer, {c->k, false, slabs, (key_depth - 1) * c->layers + layer},
                           {c->v, false, slabs, (value_depth - 1) * c->layers + layer}, prefix_len,
                           block_len, max_block, q, k_blk, v_blk, num_q_heads, softmax_scale, out,
-                          lse, workspace, workspace_bytes, stream);
+                          lse, workspace, workspace_bytes, clear_status, stream);
 }
+
+namespace {
 
 // Depth d of a das_kv_cache_f8: d = R is the bf16 top tensor (slab = layer),
 // d < R the e4m3 low tensor (slab (d - 1) * layers + layer).
@@ -266,7 +274,7 @@ das_status attention_f8(const das_kv_cache_f8 *c, int layer, int key_depth, int 
     return attention_core(sh, layer, f8_operand(c, c->k_top, c->k_low, key_depth, layer),
                           f8_operand(c, c->v_top, c->v_low, value_depth, layer), prefix_len,
                           block_len, max_block, q, k_blk, v_blk, num_q_heads, softmax_scale, out,
-                          lse, workspace, workspace_bytes, stream);
+                          lse, workspace, workspace_bytes, false, stream);
 }
 
 }  // namespace
@@ -294,7 +302,7 @@ das_status das_mature_v_attention(const das_kv_cache *cache, int layer, int key_
                                   size_t workspace_bytes, void *stream) {
     return das::attention(cache, layer, key_depth, value_depth, prefix_len, block_len, max_block,
                           q, k_blk, v_blk, num_q_heads, softmax_scale, out, lse, workspace,
-                          workspace_bytes, stream);
+                          workspace_bytes, false, stream);
 }
 
 das_status das_verify_attention(const das_kv_cache *cache, int layer, int depth,
@@ -305,7 +313,7 @@ das_status das_verify_attention(const das_kv_cache *cache, int layer, int depth,
                                 void *stream) {
     return das::attention(cache, layer, depth, depth, prefix_len, block_len, max_block, q, k_blk,
                           v_blk, num_q_heads, softmax_scale, out, lse, workspace, workspace_bytes,
-                          stream);
+                          false, stream);
 }
 
 das_status das_greedy_accept(const float *logits, const int32_t *draft_ids, int B, int W,

@@ -55,6 +55,16 @@ cudaError_t attn_launch(const AttnParams &p, int head_dim, bool keys_e4m3, bool 
                         const CUtensorMap &tm_kb, const CUtensorMap &tm_vb,
                         const CUtensorMap &tm_q, cudaStream_t stream);
 
+// das_mature_v_attention (key_depth = value_depth for the verify attention)
+// with every argument checked; with clear_status, the workspace's 256-byte
+// header is zeroed on `stream` after the checks pass, right before the
+// launch (nothing is enqueued for a call that returns an error).
+das_status attention(const das_kv_cache *c, int layer, int key_depth, int value_depth,
+                     const int32_t *prefix_len, const int32_t *block_len, int max_block,
+                     const void *q, const void *k_blk, const void *v_blk, int num_q_heads,
+                     float softmax_scale, void *out, float *lse, void *workspace,
+                     size_t workspace_bytes, bool clear_status, void *stream);
+
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream);

@@ -12,7 +12,14 @@
 // The scratch is shared by every call on a device, so calls that overlap in
 // time on the GPU (on different streams) race on it; callers must order
 // them.  Its contents persist between calls; the only part that must start at
-// zero (the status word at its head) is cleared by every call.
+// zero (the status word at its head) is cleared by every call that passes
+// its argument checks, just before its kernels are launched.
+//
+// The array's device address is looked up once per device (a host-side name
+// of a __device__ variable is not a device address) and kept for the
+// process; a call after the device's primary context was destroyed
+// (cudaDeviceReset) would use a stale address, so such a reset ends the use
+// of this entry point in that process.
 #include <mutex>
 
 #include "das_internal.h"
@@ -49,18 +56,28 @@ extern "C" das_status das_mature_v_attention_noalloc(
     const size_t need = das_workspace_size(cache, num_q_heads, max_block);
     if (need > kScratchBytes) return DAS_ERR_WORKSPACE;
     if (need == 0)  // unsupported or invalid shape: let the full check report it
-        return das_mature_v_attention(cache, layer, key_depth, value_depth, prefix_len,
-                                      block_len, max_block, q, k_blk, v_blk, num_q_heads,
-                                      softmax_scale, out, lse, nullptr, 0, stream);
+        return das::attention(cache, layer, key_depth, value_depth, prefix_len, block_len,
+                              max_block, q, k_blk, v_blk, num_q_heads, softmax_scale, out, lse,
+                              nullptr, 0, false, stream);
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return DAS_ERR_CUDA;
     void *ws = scratch_address(dev);
     if (!ws) return DAS_ERR_CUDA;
-    // the status word must start at zero for this call
-    if (cudaMemsetAsync(ws, 0, das::kWorkspaceHeader, static_cast<cudaStream_t>(stream)) !=
-        cudaSuccess)
-        return DAS_ERR_CUDA;
-    return das_mature_v_attention(cache, layer, key_depth, value_depth, prefix_len, block_len,
-                                  max_block, q, k_blk, v_blk, num_q_heads, softmax_scale, out, lse,
-                                  ws, kScratchBytes, stream);
+    // the status word must start at zero for this call: the attention path
+    // clears it once every argument has been checked, just before its launch
+    return das::attention(cache, layer, key_depth, value_depth, prefix_len, block_len, max_block,
+                          q, k_blk, v_blk, num_q_heads, softmax_scale, out, lse, ws, kScratchBytes,
+                          true, stream);
+}
+
+extern "C" das_status das_noalloc_status(int32_t *dst, void *stream) {
+    if (!dst) return DAS_ERR_INVALID_ARG;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return DAS_ERR_CUDA;
+    void *ws = scratch_address(dev);
+    if (!ws) return DAS_ERR_CUDA;
+    return cudaMemcpyAsync(dst, ws, sizeof(int32_t), cudaMemcpyDefault,
+                           static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAS_OK
+               : DAS_ERR_CUDA;
 }
