@@ -1,5 +1,8 @@
 """Helpers shared by the GPU tests: device upload of generator output, the
 oracle comparison and the tolerance of the float outputs."""
+import json
+import os
+
 import numpy as np
 import torch
 
@@ -7,13 +10,15 @@ import oracle
 import synth
 from synth import workloads as wl_mod
 
-# Tolerances: bf16 outputs max abs 1e-2 (relative to max(1, |o|) above 1,
-# where bf16 spacing alone exceeds it) and max rel 1e-2, fp32 LSE max abs
-# 1e-4.  The relative error of an element is taken against the larger of its
-# own magnitude and the RMS of its reference row (the head_dim values of one
-# query row): the kernel rounds the softmax weights P to bf16 for the tensor-
-# core P.V product (relative error <= 2^-9 per weight), which perturbs an
-# output by a fraction of the row's scale, not of the element itself.
+# Tolerances (stated for the method's bf16 outputs and fp32 lse): every
+# element's raw error |g - o| <= 1e-2, plus half a bf16 ulp of |o| where
+# |o| >= 4 (there the rounding of the output to bf16 alone, up to half an ulp
+# = 2^-6 in [4, 8), can exceed 1e-2; below 4 it is at most 2^-7 in [2, 4),
+# under 1e-2, and the raw bound holds as stated); relative error <= 1e-2 against the larger
+# of |o| and the RMS of the reference row (the head_dim values of one query
+# row: the kernel rounds the softmax weights P to bf16 for the tensor-core
+# P.V product, relative error <= 2^-9 per weight, which perturbs an output by
+# a fraction of the row's scale, not of the element); lse max abs 1e-4.
 OUT_ABS, OUT_REL, LSE_ABS = 1e-2, 1e-2, 1e-4
 
 
@@ -35,23 +40,62 @@ def host_bits(t):
     return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
 
 
+def half_ulp_bf16(o):
+    """Half the bf16 spacing at |o| (8 significant bits): 2^(e - 8) for |o| in
+    [2^e, 2^(e+1)); 0 at 0."""
+    a = np.abs(np.asarray(o, dtype=np.float64))
+    e = np.floor(np.log2(np.where(a > 0, a, 1.0)))
+    return np.where(a > 0, np.exp2(e - 8), 0.0)
+
+
+def abs_bound(o):
+    """Allowed raw error per element: 1e-2, plus half a bf16 ulp where |o| >= 4."""
+    return OUT_ABS + np.where(np.abs(o) >= 4.0, half_ulp_bf16(o), 0.0)
+
+
+def parity_errors(out_gpu, out_ref, lse_gpu=None, lse_ref=None):
+    """(max raw abs error, max relative error, max lse error or None)."""
+    g = np.asarray(out_gpu, dtype=np.float64)
+    o = np.asarray(out_ref, dtype=np.float64)
+    err = np.abs(g - o)
+    lse_err = None
+    if lse_gpu is not None:
+        lg = np.asarray(lse_gpu, dtype=np.float64)
+        lo = np.asarray(lse_ref, dtype=np.float64)
+        fin = ~np.isneginf(lo)
+        lse_err = float(np.abs(lg[fin] - lo[fin]).max(initial=0.0))
+    return float(err.max(initial=0.0)), float((err / rel_denominator(o)).max(initial=0.0)), lse_err
+
+
+def record_parity(where, abs_err, rel_err, lse_err):
+    """Print one parity case's measured errors; with PARITY_LOG set, also
+    append them as a JSON line to that file."""
+    print(f"parity {where}: max abs {abs_err:.3e} max rel {rel_err:.3e} "
+          f"lse {lse_err if lse_err is None else f'{lse_err:.3e}'}")
+    path = os.environ.get("PARITY_LOG")
+    if path:
+        with open(path, "a") as f:
+            f.write(json.dumps({"case": where, "max_abs": abs_err, "max_rel": rel_err,
+                                "lse_max_abs": lse_err}) + "\n")
+
+
 def assert_close(out_gpu, out_ref, lse_gpu=None, lse_ref=None, where=""):
     g = np.asarray(out_gpu, dtype=np.float64)
     o = np.asarray(out_ref, dtype=np.float64)
     assert np.all(np.isfinite(g)), f"non-finite output {where}"
     err = np.abs(g - o)
-    rel = err / rel_denominator(o)
-    # abs error against max(1, |o|): bf16 spacing alone is 2^-7 at |o| = 2
-    scaled = err / np.maximum(np.abs(o), 1.0)
-    assert scaled.max(initial=0) <= OUT_ABS, f"max abs {err.max():.3e} {where}"
-    assert rel.max(initial=0) <= OUT_REL, f"max rel {rel.max():.3e} {where}"
+    a, r, le = parity_errors(g, o, lse_gpu, lse_ref)
+    record_parity(where, a, r, le)
+    worst = np.unravel_index(np.argmax(err - abs_bound(o)), err.shape) if err.size else ()
+    assert np.all(err <= abs_bound(o)), \
+        f"max abs {a:.3e} (worst over bound at {worst}: |o| = {abs(o[worst]) if err.size else 0:.3f}) {where}"
+    assert r <= OUT_REL, f"max rel {r:.3e} {where}"
     if lse_gpu is not None:
         lg = np.asarray(lse_gpu, dtype=np.float64)
         lo = np.asarray(lse_ref, dtype=np.float64)
         inf = np.isneginf(lo)
         assert np.array_equal(np.isneginf(lg), inf), f"lse -inf pattern differs {where}"
-        d = np.abs(lg[~inf] - lo[~inf])
-        assert d.max(initial=0) <= LSE_ABS, f"lse max abs {d.max(initial=0):.3e} {where}"
+        assert le <= LSE_ABS, f"lse max abs {le:.3e} {where}"
 
 
 def run_small(wl, layer=0, key_depth=None, value_depth=None, prefix=None, block=None,

@@ -13,9 +13,11 @@ one prompt token changes the whole continuation).
 
 Two implementations of the same model:
   ToyLoopedCPU  fp64 numpy, attention by the oracle (test infrastructure);
-  ToyLoopedGPU  fp32 torch for the projections, attention, acceptance and the
-                commit through the library (das_verify_attention,
-                das_greedy_accept, das_kv_append).
+  ToyLoopedGPU  fp64 torch on the GPU for the projections (so q, k, v round
+                to the same bf16 values as on the CPU while the hidden
+                states agree), attention, acceptance and the commit through
+                the library (das_verify_attention, das_greedy_accept,
+                das_kv_append).
 Both decode autoregressively (ar) or speculatively (spec: a block [anchor,
 y_1 .. y_{w-1}] verified in one pass, the longest agreeing prefix accepted,
 n = min(a + 1, w) inputs committed)."""
@@ -89,7 +91,7 @@ class ToyLoopedGPU:
 
         import paper_2609_34538_gb300 as das
         self.t, self.das, self.w, self.cap = torch, das, w, cap
-        f = lambda a: torch.tensor(a, dtype=torch.float32, device="cuda")
+        f = lambda a: torch.tensor(a, dtype=torch.float64, device="cuda")
         self.E, self.Wq, self.Wk, self.Wv, self.Wo, self.U = map(
             f, (w.E, w.Wq, w.Wk, w.Wv, w.Wo, w.U))
         self.cache = das.DepthKVCache.empty(w.R, w.L, 1, cap, w.H, w.D)
@@ -110,13 +112,15 @@ class ToyLoopedGPU:
         sv = t.empty_like(sk)
         for r in range(1, w.R + 1):
             for l in range(w.L):
-                q = (h @ self.Wq[l]).to(t.bfloat16).view(1, T, w.H, w.D)
-                sk[r - 1, l] = (h @ self.Wk[l]).to(t.bfloat16).view(1, T, w.H, w.D)
-                sv[r - 1, l] = (h @ self.Wv[l]).to(t.bfloat16).view(1, T, w.H, w.D)
+                # fp64 -> fp32 -> bf16, the rounding path of the CPU model
+                bf = lambda x: x.float().to(t.bfloat16).view(1, T, w.H, w.D)
+                q = bf(h @ self.Wq[l])
+                sk[r - 1, l] = bf(h @ self.Wk[l])
+                sv[r - 1, l] = bf(h @ self.Wv[l])
                 out, _ = das.das_verify_attention(self.cache, l, r, self.pl, bl, q, sk[r - 1, l],
                                                   sv[r - 1, l], self.ws[T])
-                h = h + t.tanh(out.float().view(T, w.H * w.D) @ self.Wo[l])
-        return (h @ self.U).contiguous(), sk, sv
+                h = h + t.tanh(out.double().view(T, w.H * w.D) @ self.Wo[l])
+        return (h @ self.U).float().contiguous(), sk, sv
 
     def accept(self, logits, draft):
         t = self.t
