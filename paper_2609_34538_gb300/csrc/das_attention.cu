@@ -33,9 +33,12 @@
 //     mask and scale them (base 2), keep a reference max m that only moves
 //     when a score exceeds it by more than 2^8 (then O and l are rescaled in
 //     TMEM), write P = 2^(s - m) as bf16 into a 128-byte-swizzled [64 rows]
-//     [64 keys] buffer (the K-major A operand of P V) and accumulate l.  At
-//     the end of a segment they read the O rows from TMEM and write O / l and
-//     the lse (or the partial).
+//     [64 keys] buffer (the K-major A operand of P V) and accumulate two row
+//     sums: of the fp32 weights (for the lse) and of the weights as rounded to
+//     bf16 (for the normalisation, so that the output is a convex combination
+//     of the values with exactly the weights the tensor core used).  At the
+//     end of a segment they read the O rows from TMEM and write O / l and the
+//     lse (or the partial).
 // The kernel is launched as a programmatic dependent of the previous kernel
 // in the stream: barrier set-up, the tensor-memory allocation, the work plan
 // (from lengths read before the wait, checked again after it) and an L2
@@ -1026,7 +1029,12 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         const bool owner = lane < 16;
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         Walk ws = w0;
-        float m_ref = -INFINITY, l_sum = 0.f;
+        // l_sum: sum of the fp32 weights 2^(s - m), for the lse; l_rnd: sum of
+        // the same weights as rounded to bf16 for the P V product, for the
+        // normalisation, so that O / l_rnd is an exact convex combination of
+        // the values (the rounding of P then moves the output by a fraction
+        // of the values' spread around it, not of the values themselves)
+        float m_ref = -INFINITY, l_sum = 0.f, l_rnd = 0.f;
         int rows_active = 0, irow = 0;
         long long seg_first = lo;
         for (long long k = 0; k < ntiles; ++k) {
@@ -1036,6 +1044,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             if (first) {
                 m_ref = -INFINITY;
                 l_sum = 0.f;
+                l_rnd = 0.f;
                 rows_active = p.G * ws.T;
                 irow = row / p.G;
                 seg_first = lo + k;
@@ -1093,6 +1102,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                     if (jump) {
                         m_ref = mt;
                         l_sum *= alpha;
+                        l_rnd *= alpha;
                     }
 #pragma unroll 1
                     for (int c = 0; c < D; c += 32) {
@@ -1151,15 +1161,25 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
-            {  // the row sum is needed only for l: after P has been handed on
-                float t16[16];
+            {  // the row sums are needed only for l: after P has been handed on
+                float t16[16], r16[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) t16[j] = v[j] + v[j + 16];
+                for (int j = 0; j < 16; ++j) {
+                    t16[j] = v[j] + v[j + 16];
+                    // word e of w holds P of keys 2e (low half) and 2e + 1
+                    const uint32_t a = w[j >> 1], b = w[(j + 16) >> 1];
+                    r16[j] = (j & 1 ? __uint_as_float(a & 0xFFFF0000u) : __uint_as_float(a << 16)) +
+                             (j & 1 ? __uint_as_float(b & 0xFFFF0000u) : __uint_as_float(b << 16));
+                }
 #pragma unroll
                 for (int wd = 8; wd > 0; wd >>= 1)
 #pragma unroll
-                    for (int j = 0; j < wd; ++j) t16[j] += t16[j + wd];
+                    for (int j = 0; j < wd; ++j) {
+                        t16[j] += t16[j + wd];
+                        r16[j] += r16[j + wd];
+                    }
                 l_sum += t16[0];
+                l_rnd += r16[0];
             }
 
             // ---- end of segment: O / l and lse ----
@@ -1171,9 +1191,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 const int pair = ws.b * p.Hkv + ws.h;
                 const size_t slot = (size_t)pair + blockIdx.x;
                 const bool write = row < rows_active;
-                // the row's sum: this thread's half plus its partner's
+                // the row's sums: this thread's half plus its partner's
                 const float l_row = l_sum + __shfl_xor_sync(kFull, l_sum, 16);
-                const float inv = l_row > 0.f ? 1.f / l_row : 0.f;
+                const float l_row_rnd = l_rnd + __shfl_xor_sync(kFull, l_rnd, 16);
+                const float inv = l_row_rnd > 0.f ? 1.f / l_row_rnd : 0.f;
                 const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;
                 const int gq = row % p.G;
                 // this thread's columns: [64 g + 32 half, +32) for each 64-column group g
