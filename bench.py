@@ -516,14 +516,17 @@ def draft_probe(name, dev, steps, warmup, peak, layers=0, compact=False):
             "steps": len(ms)}
 
 
-def commit_probe(name, dev, steps, warmup, peak, layers=0):
+def commit_probe(name, dev, steps, warmup, peak, layers=0, calls=4):
     """Greedy acceptance and the commit at a verify-and-commit workload's
-    shape (Sec. 3.4, App. B.1), each timed on its own (a CUDA graph of one
-    call, L2 flushed before every step): accept over fp32 logits [B][w][vocab]
-    with planted acceptance lengths, then the append of n_b = min(a_b + 1, w)
-    staged inputs' K/V at all R depths and L layers into the full cache.
-    Algorithmic bytes: accept B * w * vocab * 4 (the logits read); append
-    2 (K and V) * sum_b n_b * R * L * Hkv * D * 2, read once and written once."""
+    shape (Sec. 3.4, App. B.1), each timed on its own as a CUDA graph of
+    `calls` back-to-back calls on distinct inputs (L2 flushed before every
+    replay; per-call time = graph time / calls): accept over fp32 logits
+    [B][w][vocab] with planted acceptance lengths, then the append of
+    n_b = min(a_b + 1, w) staged inputs' K/V at all R depths and L layers
+    into the full cache (each call appends after the previous one).
+    Algorithmic bytes per call: accept B * w * vocab * 4 (the logits read);
+    append 2 (K and V) * sum_b n_b * R * L * Hkv * D * 2, read once and
+    written once."""
     import torch
 
     import paper_2609_34538_gb300 as das
@@ -534,12 +537,15 @@ def commit_probe(name, dev, steps, warmup, peak, layers=0):
     if layers:
         wl = wl.replace(layers=layers)
     W, B = wl.max_block, wl.batch
+    wl = wl.replace(extra_capacity=(calls - 1) * W)
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
         K, V = sdev.build_cache(wl, key_depths=[], value_depths=[], device=dev)
         cache = das.DepthKVCache(K, V)
-        kn, vn = sdev.build_staged(wl, W, device=dev)
+        staged = [sdev.build_staged(wl.replace(seed=wl.seed + c), W, device=dev)
+                  for c in range(calls)]
         a_star, draft, logits = sdev.accept_tensors(wl, dev)
+        logit_bufs = [logits] + [logits.clone() for _ in range(calls - 1)]
         P0 = torch.from_numpy(wl.prefix_lens()).to(dev)
         pl = P0.clone()
         acc = torch.empty(B, dtype=torch.int32, device=dev)
@@ -548,8 +554,15 @@ def commit_probe(name, dev, steps, warmup, peak, layers=0):
         flag = torch.zeros(1, dtype=torch.int32, device=dev)
         flush = torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev)
     stream.synchronize()
-    accept = lambda: das.das_greedy_accept(logits, draft, acc, tid, nxt, stream=stream)
-    append = lambda: das.das_kv_append(cache, kn, vn, acc, pl, flag, stream=stream)
+
+    def accept():
+        for lg in logit_bufs:
+            das.das_greedy_accept(lg, draft, acc, tid, nxt, stream=stream)
+
+    def append():
+        for kn, vn in staged:
+            das.das_kv_append(cache, kn, vn, acc, pl, flag, stream=stream)
+
     with torch.cuda.stream(stream):
         accept()
         append()
@@ -573,26 +586,27 @@ def commit_probe(name, dev, steps, warmup, peak, layers=0):
             graphs[1].replay()
             e[2].record(stream)
     stream.synchronize()
-    if not (np.array_equal(acc.cpu().numpy(), a_star) and int(flag.item()) == 0):
-        raise SystemExit("bench: accept / append results failed their checks")
-    acc_ms = [e[0].elapsed_time(e[1]) for e in ev[warmup:]]
-    app_ms = [e[1].elapsed_time(e[2]) for e in ev[warmup:]]
     n = np.minimum(a_star.astype(np.int64) + 1, W)
+    if not (np.array_equal(acc.cpu().numpy(), a_star) and int(flag.item()) == 0
+            and np.array_equal(pl.cpu().numpy(), wl.prefix_lens() + calls * n)):
+        raise SystemExit("bench: accept / append results failed their checks")
+    acc_ms = [e[0].elapsed_time(e[1]) / calls for e in ev[warmup:]]
+    app_ms = [e[1].elapsed_time(e[2]) / calls for e in ev[warmup:]]
     acc_bytes = B * W * logits.shape[2] * 4
     app_bytes = 2 * int(n.sum()) * wl.depths * wl.layers * wl.kv_heads * wl.head_dim * 2 * 2
-    del K, V, cache, kn, vn, flush
+    del K, V, cache, staged, logit_bufs, flush
     torch.cuda.empty_cache()
 
     def rate(nbytes, ms):
         t = statistics.mean(ms)
         gbs = nbytes / (t / 1e3) / 1e9
-        return {"us": round(t * 1e3, 2), "bytes": nbytes, "gbs": round(gbs, 1),
+        return {"us_per_call": round(t * 1e3, 2), "bytes_per_call": nbytes, "gbs": round(gbs, 1),
                 "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peak,
                              "unit": "GB/s", "frac": round(gbs / peak, 4)}}
 
-    return {"workload": wl.name,
+    return {"workload": wl.name, "calls_per_graph": calls,
             "accept": {"shape": [B, W, int(logits.shape[2])], **rate(acc_bytes, acc_ms)},
-            "append": {"positions_committed": int(n.sum()), "depths": wl.depths,
+            "append": {"positions_committed_per_call": int(n.sum()), "depths": wl.depths,
                        "layers": wl.layers, **rate(app_bytes, app_ms)},
             "steps": len(acc_ms)}
 

@@ -16,23 +16,22 @@ namespace das {
 namespace {
 
 // ---- greedy acceptance and the DAS-Wave readout ------------------------------
-// One cluster of CTAS CTAs per sequence (CTAS = 16 for up to four sequences,
-// which spreads a sequence's logits over more SMs, else 8: with more
-// sequences, 16-CTA clusters measured slower than 8-CTA ones).  CTA r of the
-// cluster scans slice r of the vocabulary for every row i < W of its sequence
-// and stores its best (value, index) per row straight into CTA 0's shared
-// memory (distributed shared memory).  The others then arrive at the cluster
-// barrier and exit; CTA 0 waits for them, reduces the CTAS candidates of each
-// row from its own shared memory and
-//   - accept mode (Sec. 3.4): writes target_ids, counts the accepted prefix
-//     and writes accepted and next_token;
-//   - readout mode (Eq. 6, Sec. 3.3): writes the argmax of row i as the guess
-//     of position i + 1, tokens[b][i + 1].
-constexpr int kAcceptThreads = 1024;
-constexpr int kAcceptWarps = kAcceptThreads / 32;
+// Two steps, neither with scratch memory beyond the outputs:
+//   row_argmax_kernel: the first maximum of every logits row, row i of
+//     sequence b scanned by k CTAs (a cluster of k, each a 1/k slice of the
+//     vocabulary, k chosen so that rows * k fills the SMs, at most 8); CTA r
+//     of the cluster stores its best (value, index) straight into CTA 0's
+//     shared memory (distributed shared memory) and CTA 0 writes
+//       accept mode (Sec. 3.4):  target_ids[b][i];
+//       readout mode (Eq. 6, Sec. 3.3):  tokens[b][i + 1];
+//   accept_scan_kernel (accept mode only, a programmatic dependent of the
+//     first): one warp per sequence finds the first mismatch between
+//     draft_ids and target_ids and writes accepted and next_token.
+constexpr int kRowThreadsMax = 1024;
+constexpr int kRowLoads = 8;    // vector loads in flight per thread
+constexpr int kMaxRowCtas = 8;  // CTAs per row: a portable cluster
 constexpr int kMaxW = 1024;
-constexpr int kBatch = 8;          // vector loads in flight per thread
-constexpr int kWideClusterMaxB = 4;  // sequences up to which a cluster has 16 CTAs
+constexpr int kScanWarps = 4;
 
 // (value, index) order of the argmax: larger value wins, equal values go to
 // the smaller index, so the result is the first maximum.
@@ -51,136 +50,132 @@ __device__ __forceinline__ void warp_best(float &bv, int &bi) {
     }
 }
 
-// dynamic shared memory of an accept CTA: candidate values [CTAS][W] and
-// indices [CTAS][W] (filled in CTA 0 by every CTA), row argmaxes [W] (CTA 0)
-__host__ __device__ constexpr size_t accept_smem_bytes(int ctas, int W) {
-    return (size_t)ctas * W * 8 + (size_t)W * 4;
-}
-
-struct ArgmaxArgs {
+struct RowArgs {
     const float *logits;  // [B][W][vocab]
-    int W, vocab, slice;
-    // accept mode
-    const int32_t *draft;
-    int32_t *accepted, *target_ids, *next_token;
-    // readout mode
-    int32_t *tokens;  // [B][stride]
+    int W, vocab, slice;  // slice: floats per CTA, a multiple of the vector width
+    int32_t *target_ids;  // accept mode: [B][W]
+    int32_t *tokens;      // readout mode: [B][stride]
     int stride;
 };
 
 // VEC = 4: float4 loads (vocab % 4 == 0 and 16-byte aligned logits), else 1.
-template <int VEC, bool READOUT, int CTAS>
-__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const ArgmaxArgs a) {
-    const float *__restrict__ logits = a.logits;
-    const int W = a.W, vocab = a.vocab, slice = a.slice;
-    extern __shared__ __align__(16) uint8_t accept_smem[];
-    float *cand_v = reinterpret_cast<float *>(accept_smem);
-    int *cand_i = reinterpret_cast<int *>(cand_v + CTAS * W);
-    int *target = cand_i + CTAS * W;
-    __shared__ float warp_v[kAcceptWarps];
-    __shared__ int warp_i[kAcceptWarps];
-    __shared__ int first_miss;
+// The cluster size k (1..8) is the launch's; row = blockIdx.x / k.
+template <int VEC, bool READOUT>
+__global__ void __launch_bounds__(kRowThreadsMax) row_argmax_kernel(const RowArgs a) {
+    __shared__ float warp_v[32];
+    __shared__ int warp_i[32];
+    __shared__ float cand_v[kMaxRowCtas];
+    __shared__ int cand_i[kMaxRowCtas];
     cg::cluster_group cluster = cg::this_cluster();
+    const int k = (int)cluster.num_blocks();
     const int rank = (int)cluster.block_rank();
-    const int b = blockIdx.x / CTAS;
+    const size_t row = blockIdx.x / k;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // a CTA's shared memory may be written by another only once that CTA has
-    // started: every CTA arrives here and waits before its first remote store
-    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // started: every CTA arrives here and waits before its remote store
+    if (k > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // the logits may come from the kernel before this one
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    float *dst_v = cluster.map_shared_rank(cand_v, 0) + rank * W;
-    int *dst_i = cluster.map_shared_rank(cand_i, 0) + rank * W;
 
-    // threads per row: the CTA's warps split over min(W, 32) rows at a time
-    int tpr = kAcceptThreads;
-    while (tpr > 32 && tpr * W > kAcceptThreads) tpr >>= 1;
-    const int rows_per_pass = kAcceptThreads / tpr, warps_per_row = tpr / 32;
-    const int lo = min(rank * slice, vocab), hi = min(lo + slice, vocab);
+    const int lo = min(rank * a.slice, a.vocab), hi = min(lo + a.slice, a.vocab);
     const int nvec = (hi - lo) / VEC;  // slice is a multiple of VEC
-    for (int i0 = 0; i0 < W; i0 += rows_per_pass) {
-        const int i = i0 + threadIdx.x / tpr;
-        const int part = threadIdx.x % tpr;
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
-        if (i < W) {
-            const float *row = logits + ((size_t)b * W + i) * (size_t)vocab + lo;
-            // batches of kBatch vector loads, all issued before the compares
-            for (int j0 = part; j0 < nvec; j0 += kBatch * tpr) {
-                float x[kBatch][VEC];
+    const float *__restrict__ src = a.logits + row * (size_t)a.vocab + lo;
+    float bv = -INFINITY;
+    int bi = 0x7fffffff;
+    const int nt = blockDim.x;
+    // batches of kRowLoads vector loads, all issued before the compares
+    for (int j0 = threadIdx.x; j0 < nvec; j0 += kRowLoads * nt) {
+        float x[kRowLoads][VEC];
 #pragma unroll
-                for (int u = 0; u < kBatch; ++u) {
-                    const int j = j0 + u * tpr;
-                    if (j < nvec) {
-                        if (VEC == 4) {
-                            const float4 y = __ldcs(reinterpret_cast<const float4 *>(row) + j);
-                            x[u][0] = y.x;
-                            x[u][1 % VEC] = y.y;
-                            x[u][2 % VEC] = y.z;
-                            x[u][VEC - 1] = y.w;
-                        } else {
-                            x[u][0] = __ldcs(row + j);
-                        }
-                    }
-                }
-#pragma unroll
-                for (int u = 0; u < kBatch; ++u) {
-                    const int j = j0 + u * tpr;
-                    if (j < nvec) {
-#pragma unroll
-                        for (int e = 0; e < VEC; ++e) better(bv, bi, x[u][e], lo + VEC * j + e);
-                    }
+        for (int u = 0; u < kRowLoads; ++u) {
+            const int j = j0 + u * nt;
+            if (j < nvec) {
+                if (VEC == 4) {
+                    const float4 y = __ldcs(reinterpret_cast<const float4 *>(src) + j);
+                    x[u][0] = y.x;
+                    x[u][1 % VEC] = y.y;
+                    x[u][2 % VEC] = y.z;
+                    x[u][VEC - 1] = y.w;
+                } else {
+                    x[u][0] = __ldcs(src + j);
                 }
             }
         }
-        warp_best(bv, bi);
-        if (lane == 0) {
-            warp_v[warp] = bv;
-            warp_i[warp] = bi;
-        }
-        __syncthreads();
-        if (i0 == 0) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
-        if (threadIdx.x < rows_per_pass && i0 + (int)threadIdx.x < W) {
-            float v = -INFINITY;
-            int y = 0x7fffffff;
-            for (int w = 0; w < warps_per_row; ++w)
-                better(v, y, warp_v[threadIdx.x * warps_per_row + w],
-                       warp_i[threadIdx.x * warps_per_row + w]);
-            dst_v[i0 + threadIdx.x] = v;
-            dst_i[i0 + threadIdx.x] = y;
-        }
-        __syncthreads();
-    }
-    // the candidates are in CTA 0 once every CTA has arrived (release); only
-    // CTA 0 waits, and no CTA's shared memory but CTA 0's is ever read remotely
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-    if (rank != 0) return;
-    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
-
-    if (threadIdx.x == 0) first_miss = W;
-    __syncthreads();
-    for (int i = threadIdx.x; i < W; i += kAcceptThreads) {
-        float v = -INFINITY;
-        int x = 0x7fffffff;
 #pragma unroll
-        for (int r = 0; r < CTAS; ++r) better(v, x, cand_v[r * W + i], cand_i[r * W + i]);
-        // a row of -inf keeps the sentinel: the first index wins
-        const int t = x == 0x7fffffff ? 0 : x;
-        if (READOUT) {
-            a.tokens[(size_t)b * a.stride + i + 1] = t;
-        } else {
-            target[i] = t;
-            a.target_ids[(size_t)b * W + i] = t;
-            if (a.draft[(size_t)b * W + i] != t) atomicMin(&first_miss, i);
+        for (int u = 0; u < kRowLoads; ++u) {
+            const int j = j0 + u * nt;
+            if (j < nvec) {
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) better(bv, bi, x[u][e], lo + VEC * j + e);
+            }
         }
     }
-    if (!READOUT) {
-        __syncthreads();
+    warp_best(bv, bi);
+    if (lane == 0) {
+        warp_v[warp] = bv;
+        warp_i[warp] = bi;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        bv = lane < (nt >> 5) ? warp_v[lane] : -INFINITY;
+        bi = lane < (nt >> 5) ? warp_i[lane] : 0x7fffffff;
+        warp_best(bv, bi);
+    }
+    if (k > 1) {
+        asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
         if (threadIdx.x == 0) {
-            const int n = first_miss;
-            a.accepted[b] = n;
-            a.next_token[b] = n < W ? target[n] : a.draft[(size_t)b * W + W - 1];
+            *cluster.map_shared_rank(cand_v + rank, 0) = bv;
+            *cluster.map_shared_rank(cand_i + rank, 0) = bi;
         }
+        // the candidates are in CTA 0 once every CTA has arrived (release);
+        // only CTA 0 waits, and only its shared memory is read remotely
+        asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+        if (rank != 0) return;
+        asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+        if (threadIdx.x == 0) {
+            bv = cand_v[0];
+            bi = cand_i[0];
+            for (int r = 1; r < k; ++r) better(bv, bi, cand_v[r], cand_i[r]);
+        }
+    }
+    if (threadIdx.x == 0) {
+        // a row of -inf keeps the sentinel: the first index wins
+        const int t = bi == 0x7fffffff ? 0 : bi;
+        if (READOUT) {
+            const size_t b = row / a.W, i = row % a.W;
+            a.tokens[b * a.stride + i + 1] = t;
+        } else {
+            a.target_ids[row] = t;
+        }
+    }
+}
+
+// accepted[b] = first i with draft[b][i] != target_ids[b][i] (W if none);
+// next_token[b] = target_ids[b][accepted[b]], or draft[b][W - 1] if all W
+// proposals were accepted.  One warp per sequence.
+__global__ void __launch_bounds__(kScanWarps * 32)
+    accept_scan_kernel(const int32_t *__restrict__ target_ids, const int32_t *__restrict__ draft,
+                       int B, int W, int32_t *__restrict__ accepted,
+                       int32_t *__restrict__ next_token) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int lane = threadIdx.x & 31;
+    const long long b = (long long)blockIdx.x * kScanWarps + (threadIdx.x >> 5);
+    if (b >= B) return;
+    const int32_t *t = target_ids + b * W, *d = draft + b * W;
+    int first = W;
+    for (int i0 = 0; i0 < W; i0 += 32) {
+        const int i = i0 + lane;
+        const unsigned m = __ballot_sync(0xffffffffu, i < W && d[i] != t[i]);
+        if (m) {
+            first = i0 + __ffs(m) - 1;
+            break;
+        }
+    }
+    if (lane == 0) {
+        accepted[b] = first;
+        next_token[b] = first < W ? t[first] : d[W - 1];
     }
 }
 
@@ -348,96 +343,36 @@ cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, unsigne
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
 }
 
-// The dynamic shared memory opt-in (and, for 16-CTA clusters, the non-portable
-// cluster size) of one accept kernel, once per device.  Returns false if the
-// kernel cannot run with that many CTAs per cluster on this device.
-template <int VEC, bool READOUT, int CTAS>
-cudaError_t accept_configure(int dev, bool &usable) {
-    static std::atomic<int> state[64];  // 0 unknown, 1 usable, 2 not usable
-    usable = false;
-    if (dev < 64) {
-        const int st = state[dev].load(std::memory_order_acquire);
-        if (st != 0) {
-            usable = st == 1;
-            return cudaSuccess;
-        }
-    }
-    auto kernel = accept_kernel<VEC, READOUT, CTAS>;
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)accept_smem_bytes(CTAS, kMaxW));
-    if (e != cudaSuccess) return e;
-    if (CTAS > 8) {
-        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-        if (e != cudaSuccess) return e;
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(CTAS);
-        cfg.blockDim = dim3(kAcceptThreads);
-        cfg.dynamicSmemBytes = accept_smem_bytes(CTAS, kMaxW);
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = CTAS;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        int clusters = 0;
-        e = cudaOccupancyMaxActiveClusters(&clusters, kernel, &cfg);
-        if (e != cudaSuccess) return e;
-        usable = clusters >= 1;
-    } else {
-        usable = true;
-    }
-    if (dev < 64) state[dev].store(usable ? 1 : 2, std::memory_order_release);
-    return cudaSuccess;
-}
-
-template <int VEC, bool READOUT, int CTAS>
-cudaError_t argmax_launch_ctas(ArgmaxArgs a, int B, cudaStream_t stream) {
-    // slices are whole float4s
-    const int slice = (a.vocab + CTAS - 1) / CTAS;
-    a.slice = (slice + 3) & ~3;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(B * CTAS));
-    cfg.blockDim = dim3(kAcceptThreads);
-    cfg.dynamicSmemBytes = accept_smem_bytes(CTAS, a.W);
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = CTAS;
-    attr[1].val.clusterDim.y = 1;
-    attr[1].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, accept_kernel<VEC, READOUT, CTAS>, a);
-}
-
+// The argmax step: k CTAs per row, k = SMs / rows clamped to [1, 8], with
+// enough threads for kRowLoads vector loads each over a 1/k slice.
 template <int VEC, bool READOUT>
-cudaError_t argmax_launch_vec(const ArgmaxArgs &a, int B, cudaStream_t stream) {
+cudaError_t row_argmax_launch(RowArgs a, long long rows, cudaStream_t stream) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    bool usable = false;
-    if (B <= kWideClusterMaxB) {
-        e = accept_configure<VEC, READOUT, 16>(dev, usable);
-        if (e != cudaSuccess) return e;
-        if (usable) return argmax_launch_ctas<VEC, READOUT, 16>(a, B, stream);
-    }
-    e = accept_configure<VEC, READOUT, 8>(dev, usable);
-    if (e != cudaSuccess) return e;
-    return argmax_launch_ctas<VEC, READOUT, 8>(a, B, stream);
+    const int sms = attn_grid_size(dev);
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    const int k = rows >= sms ? 1 : (int)std::min<long long>(kMaxRowCtas, sms / rows);
+    const int slice = (a.vocab + k - 1) / k;
+    a.slice = (slice + VEC - 1) / VEC * VEC;
+    const int nvec = a.slice / VEC;
+    int threads = (nvec + kRowLoads - 1) / kRowLoads;
+    threads = std::max(32, std::min(kRowThreadsMax, (threads + 31) / 32 * 32));
+    if (rows * k > 0x7fffffffLL) return cudaErrorInvalidValue;
+    return launch_pdl(row_argmax_kernel<VEC, READOUT>, dim3((unsigned)(rows * k)),
+                      dim3((unsigned)threads), (unsigned)k, stream, a);
 }
 
-cudaError_t argmax_launch(const ArgmaxArgs &a, int B, bool readout, cudaStream_t stream) {
+cudaError_t argmax_launch(const RowArgs &a, int B, bool readout, cudaStream_t stream) {
     if (B == 0) return cudaSuccess;
-    if (a.W < 1 || a.W > kMaxW || B > 0x7fffffff / 16) return cudaErrorInvalidValue;
+    if (a.W < 1 || a.W > kMaxW) return cudaErrorInvalidValue;
+    const long long rows = (long long)B * a.W;
     const bool vec = (a.vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(a.logits) & 15u) == 0;
     if (readout)
-        return vec ? argmax_launch_vec<4, true>(a, B, stream)
-                   : argmax_launch_vec<1, true>(a, B, stream);
-    return vec ? argmax_launch_vec<4, false>(a, B, stream)
-               : argmax_launch_vec<1, false>(a, B, stream);
+        return vec ? row_argmax_launch<4, true>(a, rows, stream)
+                   : row_argmax_launch<1, true>(a, rows, stream);
+    return vec ? row_argmax_launch<4, false>(a, rows, stream)
+               : row_argmax_launch<1, false>(a, rows, stream);
 }
 
 }  // namespace
@@ -445,20 +380,21 @@ cudaError_t argmax_launch(const ArgmaxArgs &a, int B, bool readout, cudaStream_t
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream) {
-    ArgmaxArgs a = {};
+    RowArgs a = {};
     a.logits = logits;
     a.W = W;
     a.vocab = vocab;
-    a.draft = draft;
-    a.accepted = accepted;
     a.target_ids = target_ids;
-    a.next_token = next_token;
-    return argmax_launch(a, B, false, stream);
+    cudaError_t e = argmax_launch(a, B, false, stream);
+    if (e != cudaSuccess || B == 0) return e;
+    return launch_pdl(accept_scan_kernel, dim3((unsigned)((B + kScanWarps - 1) / kScanWarps)),
+                      dim3(kScanWarps * 32), 1, stream, static_cast<const int32_t *>(target_ids),
+                      draft, B, W, accepted, next_token);
 }
 
 cudaError_t wave_readout_launch(const float *logits, int B, int W, int vocab, int32_t *tokens,
                                 int stride, cudaStream_t stream) {
-    ArgmaxArgs a = {};
+    RowArgs a = {};
     a.logits = logits;
     a.W = W;
     a.vocab = vocab;

@@ -56,21 +56,29 @@ def test_accept_ties_and_infinities():
     assert list(acc) == [4, 3, 3]
 
 
-@pytest.mark.parametrize("B", [1, 8])
-def test_accept_ties_across_slices(B):
-    """Equal maxima in two CTAs' vocabulary slices: a sequence is scanned by
-    16 CTAs (slices of 260 columns at V = 4099) for up to four sequences and
-    by 8 (slices of 516) beyond; the smaller index wins either way."""
-    W, V = 3, 4099
+@pytest.mark.parametrize("B", [1, 8, 32])
+@pytest.mark.parametrize("V", [4099, 4096])
+def test_accept_ties_across_slices(B, V):
+    """Equal maxima on both sides of a boundary between two CTAs' vocabulary
+    slices: a row is scanned by k CTAs (k = SMs / rows, 1..8; slices of
+    ceil(V / k) columns, rounded up to whole float4s when V % 4 == 0).  Row
+    k - 2 of every sequence holds a tie straddling the boundary of a k-way
+    split, so whatever k the launch picks, some row's tie crosses CTAs; the
+    smaller index wins either way."""
+    W = 7
     logits = np.zeros((B, W, V), dtype=np.float32)
-    logits[:, 0, [259, 260]] = 5.0
-    logits[:, 1, [515, 516]] = 5.0
-    logits[:, 2, [V - 1, 0]] = 5.0
     draft = np.zeros((B, W), dtype=np.int32)
-    draft[:, 0], draft[:, 1] = 259, 515
+    first = []
+    for r in range(W):
+        k = r + 2
+        s = -(-V // k)
+        if V % 4 == 0:
+            s = -(-s // 4) * 4
+        logits[:, r, [s - 1, s]] = 5.0
+        draft[:, r] = s - 1
+        first.append(s - 1)
     acc, tid, _ = check_accept(logits, draft)
-    assert np.all(tid[:, 0] == 259) and np.all(tid[:, 1] == 515) and np.all(tid[:, 2] == 0)
-    assert np.all(acc == 3)
+    assert np.all(tid == np.array(first)[None, :]) and np.all(acc == W)
 
 
 def _append_case(R, L, B, cap, H, D, W, pl, acc, seed):
