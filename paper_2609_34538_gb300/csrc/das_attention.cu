@@ -152,6 +152,13 @@ __device__ __forceinline__ void tma_prefetch_5d(const CUtensorMap *map, int c0, 
                  "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
                  : "memory");
 }
+__device__ __forceinline__ void tma_prefetch_4d(const CUtensorMap *map, int c0, int c1, int c2,
+                                                int c3) {
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
 __device__ __forceinline__ void tma_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0,
                                        int c1, int c2, int c3) {
     asm volatile(
@@ -739,6 +746,12 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         // this one writes them, the loads after the wait still see its data).
         if (warp == kProducerWarp && elect_one()) {
             Walk wp = w0;
+            // the first segment's query rows (the kernel before this one may
+            // be the one writing them: a prefetch only warms L2)
+            if (ntiles > 0)
+#pragma unroll
+                for (int dp = 0; dp < Lt::kPanels; ++dp)
+                    tma_prefetch_4d(&tm_q, dp * 64, wp.h * p.G, 0, wp.b);
             for (long long j = 0; j < ntiles && j < kPrefetchTiles && wp.t < wp.nt - 1; ++j) {
                 const int tok = wp.t * kTileKeys;
 #pragma unroll
