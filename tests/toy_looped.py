@@ -35,22 +35,31 @@ def bf16_bits_to_f64(b):
 
 
 class Weights:
-    def __init__(self, seed, V=64, d=32, H=2, D=64, L=2, R=4):
+    """qk / v: scales of the query-key and value projections (relative to
+    1/sqrt(d)); larger qk sharpens attention and makes the continuation more
+    sensitive to small changes of the attention outputs."""
+
+    def __init__(self, seed, V=64, d=32, H=2, D=64, L=2, R=4, qk=2.0, v=1.0):
         rng = np.random.default_rng(seed)
         self.V, self.d, self.H, self.D, self.L, self.R = V, d, H, D, L, R
         self.E = rng.normal(0, 1, (V, d))
         s = 1.0 / np.sqrt(d)
-        self.Wq = rng.normal(0, 2 * s, (L, d, H * D))
-        self.Wk = rng.normal(0, 2 * s, (L, d, H * D))
-        self.Wv = rng.normal(0, s, (L, d, H * D))
+        self.Wq = rng.normal(0, qk * s, (L, d, H * D))
+        self.Wk = rng.normal(0, qk * s, (L, d, H * D))
+        self.Wv = rng.normal(0, v * s, (L, d, H * D))
         self.Wo = rng.normal(0, 1.0 / np.sqrt(H * D), (L, H * D, d))
         self.U = np.random.default_rng(seed + 100).normal(0, 1, (d, V))
 
 
 class ToyLoopedCPU:
-    def __init__(self, w, cap):
+    """bf16_outputs: round every attention output to bf16 (the library's
+    output type) before the residual update, to measure how much that
+    rounding alone moves the logits."""
+
+    def __init__(self, w, cap, bf16_outputs=False):
         import oracle
         self.o, self.w, self.cap = oracle, w, cap
+        self.bf16_outputs = bf16_outputs
         shape = (w.R, w.L, 1, cap, w.H, w.D)
         self.K = np.zeros(shape, np.uint16)
         self.V = np.zeros(shape, np.uint16)
@@ -70,6 +79,8 @@ class ToyLoopedCPU:
                 sk[r - 1, l], sv[r - 1, l] = k, v
                 out, _ = self.o.attention(self.K, self.V, l, r, r, np.array([self.P], np.int32),
                                           np.array([T], np.int32), q, k, v)
+                if self.bf16_outputs:
+                    out = bf16_bits_to_f64(to_bf16_bits(out))
                 h = h + np.tanh(out[0].reshape(T, w.H * w.D) @ w.Wo[l])
         return (h @ w.U).astype(np.float32), sk, sv
 
@@ -147,9 +158,10 @@ def prefill(m, prompt):
     return prompt[-1]
 
 
-def ar(m, prompt, n, margins=None):
+def ar(m, prompt, n, margins=None, logits_out=None):
     """Greedy AR decoding; if `margins` is a list, the gap between the two
-    largest logits of every step is appended to it."""
+    largest logits of every step is appended to it; if `logits_out` is a
+    list, every step's logits (float64) are."""
     anchor, out = prefill(m, prompt), []
     while len(out) < n:
         logits, sk, sv = m.forward([anchor])
@@ -157,10 +169,13 @@ def ar(m, prompt, n, margins=None):
         m.commit(sk, sv, 0)                   # the anchor is materialized
         out.append(int(tid[0]))
         anchor = out[-1]
+        row = np.asarray(logits[0].cpu() if hasattr(logits, "cpu") else logits[0],
+                         dtype=np.float64)
         if margins is not None:
-            row = np.sort(np.asarray(logits[0].cpu() if hasattr(logits, "cpu") else logits[0],
-                                     dtype=np.float64))
-            margins.append(row[-1] - row[-2])
+            srt = np.sort(row)
+            margins.append(srt[-1] - srt[-2])
+        if logits_out is not None:
+            logits_out.append(row)
     return out
 
 
