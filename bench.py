@@ -427,7 +427,7 @@ def gpu_arm(args):
         "sequential_draft": seq,
         "das_wave_refinement": wave,
         "e4m3_cache_draft": f8,
-        "gpu_launches": K_steps * (2 * L * 2 + 1 + 2),
+        "gpu_launches": K_steps * (2 * L * 2 + 2 + 2),
         "e2e": e2e,
         "cpu_baseline": cpu,
         "clocks": clocks.summary(),

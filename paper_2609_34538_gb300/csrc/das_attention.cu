@@ -369,14 +369,17 @@ __device__ __forceinline__ void walk_next(const AttnParams &p, Walk &w) {
 }
 
 // Extra weight of a pair's block tile when the list is split.  Ending one
-// segment (the mostly empty block tile holding a pipeline slot, the wait for
-// the last P V, the partial write) costs a CTA about two tiles' time, so a
-// range that holds a block tile takes two tiles fewer while there is at
-// least one CTA per pair; with more pairs than CTAs nearly every range holds
-// one and the weight would only move work around (weights 1-3 and CTA-per-
-// pair thresholds 1 and 4 measured on the decode, long, batched and verify
-// workloads).
-constexpr int kBlockWeight = 2;
+// segment and starting the next (the mostly empty block tile holding a
+// pipeline slot, the wait for the last P V, the partial write, the next
+// queries) costs a CTA two to three tiles' time (a fit of per-CTA loop times
+// on the batched workload: about 1.1 us per block tile plus 0.65 us per
+// segment, against 0.72 us per tile), so a range that holds a block tile
+// takes three tiles fewer while there is at least one CTA per pair; with
+// more pairs than CTAs nearly every range holds one and the weight would
+// only move work around (weights 1-4 and CTA-per-pair thresholds 1 and 4
+// measured on the decode, long, batched and verify workloads; 3 against 2:
+// long 86.9 -> 86.7 us, the others within 0.1 %).
+constexpr int kBlockWeight = 3;
 constexpr int kCtasPerPairForWeight = 1;
 
 // The split of the tile list: tile x of pair q has weighted position

@@ -69,11 +69,11 @@ def test_split_across_many_ctas():
     run_small(small(batch=2, kv_heads=2, q_heads=8, prefix=(5000, 5000), block=(8,)))
 
 
-@pytest.mark.parametrize("P", [4608, 4609, 9000])
+@pytest.mark.parametrize("P", [5760, 5761, 9000])
 def test_weighted_split_threshold(P):
-    """8 pairs on 152 CTAs: the split weights block tiles (weight 2) once the
-    weighted list holds at least (2 + 2) positions per CTA,
-    8 (ceil(P / 64) + 1) + 2 * 8 >= 4 * 152, i.e. P >= 4609; both sides of
+    """8 pairs on 152 CTAs: the split weights block tiles (extra weight 3)
+    once the weighted list holds at least (2 + 3) positions per CTA,
+    8 (ceil(P / 64) + 1) + 3 * 8 >= 5 * 152, i.e. P >= 5761; both sides of
     the threshold."""
     run_small(small(batch=1, kv_heads=8, q_heads=8, prefix=(P, P), block=(8,)))
 
