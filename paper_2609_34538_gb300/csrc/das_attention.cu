@@ -1289,28 +1289,36 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
 }  // namespace
 
 // ---- split-K merge ------------------------------------------------------------
-// One warp per query row of a split pair; lane l holds columns [VPL l,
-// VPL (l+1)).  With partial s holding O_s / l_s and lse_s for the row:
+// One warp per RPW query rows of a split pair (rows w, w + 4, ... of the
+// CTA's 4 RPW rows); lane l holds columns [VPL l, VPL (l+1)).  With partial s
+// holding O_s / l_s and lse_s for the row:
 //   out = sum_s e^(lse_s - M) O_s / l_s / sum_s e^(lse_s - M),
 //   lse = M + ln sum_s e^(lse_s - M),  M = max_s lse_s,
 // and rows past the block get 0 and lse -inf.  The pair's segments are found
 // from the lengths before griddepcontrol.wait (the attention grid this one
 // depends on started after every kernel that could write them had
-// completed); the partials are read after it, SEGS segments' loads in
-// flight.  SEGS trades round trips for registers: at D = 128, 8 segments take
-// 116 registers a thread (4 CTAs per SM), 4 take 72 (7), 2 take 40 (12).
+// completed); the partials are read after it, SEGS segments of each of the
+// RPW rows in flight at once.  SEGS x RPW trades round trips and CTAs for
+// registers: at D = 128, 8 x 1 takes 116 registers a thread (4 CTAs per SM),
+// 4 x 1 72 (7), 2 x 1 40 (12), 2 x 2 about the same as 4 x 1 with half the
+// CTAs.
 constexpr int kMergeWarps = 4;
 
-template <int D, int SEGS>
-__global__ void __launch_bounds__(kMergeWarps * 32, SEGS == 2 ? 12 : SEGS == 4 ? 7 : 4)
+template <int SEGS, int RPW>
+constexpr int merge_min_blocks() {
+    return SEGS * RPW >= 8 ? 4 : SEGS * RPW >= 4 ? 7 : 12;
+}
+
+template <int D, int SEGS, int RPW>
+__global__ void __launch_bounds__(kMergeWarps * 32, merge_min_blocks<SEGS, RPW>())
     merge_kernel(const AttnParams p) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     constexpr int VPL = D / 32;
-    constexpr int kSegs = SEGS;
-    const int rblocks = (p.rows_max + kMergeWarps - 1) / kMergeWarps;
+    constexpr int kRowsPerCta = kMergeWarps * RPW;
+    const int rblocks = (p.rows_max + kRowsPerCta - 1) / kRowsPerCta;
     const int pair = blockIdx.x / rblocks;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int row = (blockIdx.x % rblocks) * kMergeWarps + warp;
+    const int row0 = (blockIdx.x % rblocks) * kRowsPerCta + warp;  // rows row0 + r * kMergeWarps
     const int b = pair / p.Hkv, h = pair % p.Hkv;
     const int C = p.num_ctas;
     // one pass: all tiles, and the tiles of the sequences before b
@@ -1334,98 +1342,126 @@ __global__ void __launch_bounds__(kMergeWarps * 32, SEGS == 2 ? 12 : SEGS == 4 ?
 
     // partials come from the attention grid
     asm volatile("griddepcontrol.wait;" ::: "memory");
-    if (nseg <= 1 || row >= p.rows_max) return;  // a single segment wrote its output
-    const int i = row / p.G, g = row % p.G;
-    uint16_t *orow =
-        p.out + (((size_t)b * p.max_block + i) * p.Hq + (size_t)h * p.G + g) * D + VPL * lane;
-    float *lrow = p.lse + ((size_t)b * p.Hq + (size_t)h * p.G + g) * p.max_block + i;
-    if (row >= rows_active) {
-        if (VPL == 4)
-            *reinterpret_cast<uint2 *>(orow) = make_uint2(0u, 0u);
-        else
-            *reinterpret_cast<uint32_t *>(orow) = 0u;
-        if (lane == 0) *lrow = -INFINITY;
-        return;
+    if (nseg <= 1) return;  // a single segment wrote its output
+    uint16_t *orow[RPW];
+    float *lrow[RPW];
+    bool act[RPW];
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+        const int row = row0 + r * kMergeWarps;
+        const int i = row / p.G, g = row % p.G;
+        orow[r] = p.out + (((size_t)b * p.max_block + i) * p.Hq + (size_t)h * p.G + g) * D +
+                  VPL * lane;
+        lrow[r] = p.lse + ((size_t)b * p.Hq + (size_t)h * p.G + g) * p.max_block + i;
+        act[r] = row < rows_active;
+        if (row < p.rows_max && !act[r]) {  // rows past the block: 0 and lse -inf
+            if (VPL == 4)
+                *reinterpret_cast<uint2 *>(orow[r]) = make_uint2(0u, 0u);
+            else
+                *reinterpret_cast<uint32_t *>(orow[r]) = 0u;
+            if (lane == 0) *lrow[r] = -INFINITY;
+        }
     }
-    float M = -INFINITY, L = 0.f, acc[VPL];
+    float M[RPW], L[RPW], acc[RPW][VPL];
 #pragma unroll
-    for (int v = 0; v < VPL; ++v) acc[v] = 0.f;
+    for (int r = 0; r < RPW; ++r) {
+        M[r] = -INFINITY;
+        L[r] = 0.f;
+#pragma unroll
+        for (int v = 0; v < VPL; ++v) acc[r][v] = 0.f;
+    }
 #pragma unroll 1
-    for (int s0 = 0; s0 < nseg; s0 += kSegs) {
-        float ls[kSegs], os[kSegs][VPL];
+    for (int s0 = 0; s0 < nseg; s0 += SEGS) {
+        float ls[RPW][SEGS], os[RPW][SEGS][VPL];
 #pragma unroll
-        for (int u = 0; u < kSegs; ++u) {
-            ls[u] = -INFINITY;
+        for (int r = 0; r < RPW; ++r)
 #pragma unroll
-            for (int v = 0; v < VPL; ++v) os[u][v] = 0.f;
-            if (s0 + u < nseg) {
-                const int c = contiguous ? c0 + s0 + u : cta_of_w(first + s0 + u, sp, C);
-                const size_t rs = ((size_t)pair + c) * p.rows_max + row;
-                ls[u] = __ldcg(p.part_lse + rs);
-                const float *src = p.part_o + rs * D + VPL * lane;
-                if (VPL == 4) {
-                    const float4 x = __ldcg(reinterpret_cast<const float4 *>(src));
-                    os[u][0] = x.x;
-                    os[u][1 % VPL] = x.y;
-                    os[u][2 % VPL] = x.z;
-                    os[u][VPL - 1] = x.w;
-                } else {
-                    const float2 x = __ldcg(reinterpret_cast<const float2 *>(src));
-                    os[u][0] = x.x;
-                    os[u][VPL - 1] = x.y;
+            for (int u = 0; u < SEGS; ++u) {
+                ls[r][u] = -INFINITY;
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) os[r][u][v] = 0.f;
+                if (act[r] && s0 + u < nseg) {
+                    const int c = contiguous ? c0 + s0 + u : cta_of_w(first + s0 + u, sp, C);
+                    const size_t rs = ((size_t)pair + c) * p.rows_max + row0 + r * kMergeWarps;
+                    ls[r][u] = __ldcg(p.part_lse + rs);
+                    const float *src = p.part_o + rs * D + VPL * lane;
+                    if (VPL == 4) {
+                        const float4 x = __ldcg(reinterpret_cast<const float4 *>(src));
+                        os[r][u][0] = x.x;
+                        os[r][u][1 % VPL] = x.y;
+                        os[r][u][2 % VPL] = x.z;
+                        os[r][u][VPL - 1] = x.w;
+                    } else {
+                        const float2 x = __ldcg(reinterpret_cast<const float2 *>(src));
+                        os[r][u][0] = x.x;
+                        os[r][u][VPL - 1] = x.y;
+                    }
                 }
             }
+#pragma unroll
+        for (int r = 0; r < RPW; ++r) {
+            float mn = M[r];
+#pragma unroll
+            for (int u = 0; u < SEGS; ++u) mn = fmaxf(mn, ls[r][u]);
+            if (mn == -INFINITY) continue;
+            const float a = __expf(M[r] - mn);  // 0 while M is -inf
+            L[r] *= a;
+#pragma unroll
+            for (int v = 0; v < VPL; ++v) acc[r][v] *= a;
+#pragma unroll
+            for (int u = 0; u < SEGS; ++u) {
+                const float wgt = __expf(ls[r][u] - mn);  // 0 for absent segments
+                L[r] += wgt;
+#pragma unroll
+                for (int v = 0; v < VPL; ++v) acc[r][v] += wgt * os[r][u][v];
+            }
+            M[r] = mn;
         }
-        float mn = M;
-#pragma unroll
-        for (int u = 0; u < kSegs; ++u) mn = fmaxf(mn, ls[u]);
-        if (mn == -INFINITY) continue;
-        const float a = __expf(M - mn);  // 0 while M is -inf
-        L *= a;
-#pragma unroll
-        for (int v = 0; v < VPL; ++v) acc[v] *= a;
-#pragma unroll
-        for (int u = 0; u < kSegs; ++u) {
-            const float wgt = __expf(ls[u] - mn);  // 0 for absent segments
-            L += wgt;
-#pragma unroll
-            for (int v = 0; v < VPL; ++v) acc[v] += wgt * os[u][v];
-        }
-        M = mn;
     }
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    if (VPL == 4)
-        *reinterpret_cast<uint2 *>(orow) = make_uint2(pack_bf16(acc[0] * inv, acc[1 % VPL] * inv),
-                                                      pack_bf16(acc[2 % VPL] * inv,
-                                                                acc[VPL - 1] * inv));
-    else
-        *reinterpret_cast<uint32_t *>(orow) = pack_bf16(acc[0] * inv, acc[VPL - 1] * inv);
-    if (lane == 0) *lrow = L > 0.f ? M + __logf(L) : -INFINITY;
+#pragma unroll
+    for (int r = 0; r < RPW; ++r) {
+        if (!act[r]) continue;
+        const float inv = L[r] > 0.f ? 1.f / L[r] : 0.f;
+        if (VPL == 4)
+            *reinterpret_cast<uint2 *>(orow[r]) =
+                make_uint2(pack_bf16(acc[r][0] * inv, acc[r][1 % VPL] * inv),
+                           pack_bf16(acc[r][2 % VPL] * inv, acc[r][VPL - 1] * inv));
+        else
+            *reinterpret_cast<uint32_t *>(orow[r]) =
+                pack_bf16(acc[r][0] * inv, acc[r][VPL - 1] * inv);
+        if (lane == 0) *lrow[r] = L[r] > 0.f ? M[r] + __logf(L[r]) : -INFINITY;
+    }
 }
 
-// Resident merge CTAs per SM for the 8-, 4- and 2-segment variants, looked
-// up once per device.
+// The merge variants (segments in flight x rows per warp) and their resident
+// CTAs per SM, looked up once per device.
+constexpr int kMergeVariants = 4;
+constexpr int kMergeSegs[kMergeVariants] = {8, 4, 2, 2};
+constexpr int kMergeRpw[kMergeVariants] = {1, 1, 1, 2};
+
 template <int D>
-cudaError_t merge_occupancy(int dev, int occ[3]) {
-    static std::atomic<int> cached[64][3];
-    if (dev < 64 && cached[dev][2].load(std::memory_order_acquire) > 0) {
-        for (int v = 0; v < 3; ++v) occ[v] = cached[dev][v].load(std::memory_order_relaxed);
+cudaError_t merge_occupancy(int dev, int occ[kMergeVariants]) {
+    static std::atomic<int> cached[64][kMergeVariants];
+    if (dev < 64 && cached[dev][kMergeVariants - 1].load(std::memory_order_acquire) > 0) {
+        for (int v = 0; v < kMergeVariants; ++v)
+            occ[v] = cached[dev][v].load(std::memory_order_relaxed);
         return cudaSuccess;
     }
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[0], merge_kernel<D, 8>,
-                                                                  kMergeWarps * 32, 0);
-    if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[1], merge_kernel<D, 4>,
-                                                          kMergeWarps * 32, 0);
-    if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[2], merge_kernel<D, 2>,
-                                                          kMergeWarps * 32, 0);
-    if (e != cudaSuccess) return e;
-    for (int v = 0; v < 3; ++v) occ[v] = std::max(occ[v], 1);
+    const void *fns[kMergeVariants] = {
+        reinterpret_cast<const void *>(merge_kernel<D, 8, 1>),
+        reinterpret_cast<const void *>(merge_kernel<D, 4, 1>),
+        reinterpret_cast<const void *>(merge_kernel<D, 2, 1>),
+        reinterpret_cast<const void *>(merge_kernel<D, 2, 2>)};
+    for (int v = 0; v < kMergeVariants; ++v) {
+        const cudaError_t e =
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ[v], fns[v], kMergeWarps * 32, 0);
+        if (e != cudaSuccess) return e;
+        occ[v] = std::max(occ[v], 1);
+    }
     if (dev < 64) {
-        cached[dev][0].store(occ[0], std::memory_order_relaxed);
-        cached[dev][1].store(occ[1], std::memory_order_relaxed);
-        cached[dev][2].store(occ[2], std::memory_order_release);
+        for (int v = 0; v < kMergeVariants - 1; ++v)
+            cached[dev][v].store(occ[v], std::memory_order_relaxed);
+        cached[dev][kMergeVariants - 1].store(occ[kMergeVariants - 1], std::memory_order_release);
     }
     return cudaSuccess;
 }
@@ -1458,31 +1494,35 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
     cfg.numAttrs = 1;
     e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8>, tk, tv, tkb, tvb, tq, p);
     if (e != cudaSuccess) return e;
-    const long long ctas = (long long)p.B * p.Hkv * ((p.rows_max + kMergeWarps - 1) / kMergeWarps);
-    cfg.gridDim = dim3((unsigned)ctas);
-    cfg.blockDim = dim3(kMergeWarps * 32);
-    cfg.dynamicSmemBytes = 0;
     // The merge variant with the fewest estimated sequential steps: waves of
     // resident merge CTAs (at least one) times L2 round trips per row (at
     // least one), for a pair's average segment count 1 + C / (B Hkv).
     const double segs = 1.0 + (double)p.num_ctas / ((double)p.B * p.Hkv);
-    int occ[3];
+    int occ[kMergeVariants];
     e = merge_occupancy<D>(dev, occ);
     if (e != cudaSuccess) return e;
-    const int seg_of[3] = {8, 4, 2};
     int best = 0;
     double best_cost = 0.0;
-    for (int v = 0; v < 3; ++v) {
+    long long best_ctas = 0;
+    for (int v = 0; v < kMergeVariants; ++v) {
+        const int rows_per_cta = kMergeWarps * kMergeRpw[v];
+        const long long ctas =
+            (long long)p.B * p.Hkv * ((p.rows_max + rows_per_cta - 1) / rows_per_cta);
         const double waves = std::max(1.0, (double)ctas / ((double)occ[v] * p.num_ctas));
-        const double cost = waves * std::max(1.0, segs / seg_of[v]);
+        const double cost = waves * std::max(1.0, segs / kMergeSegs[v]);
         if (v == 0 || cost < best_cost) {
             best = v;
             best_cost = cost;
+            best_ctas = ctas;
         }
     }
-    if (best == 0) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 8>, p);
-    if (best == 1) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 4>, p);
-    return cudaLaunchKernelEx(&cfg, merge_kernel<D, 2>, p);
+    cfg.gridDim = dim3((unsigned)best_ctas);
+    cfg.blockDim = dim3(kMergeWarps * 32);
+    cfg.dynamicSmemBytes = 0;
+    if (best == 0) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 8, 1>, p);
+    if (best == 1) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 4, 1>, p);
+    if (best == 2) return cudaLaunchKernelEx(&cfg, merge_kernel<D, 2, 1>, p);
+    return cudaLaunchKernelEx(&cfg, merge_kernel<D, 2, 2>, p);
 }
 
 }  // namespace tc

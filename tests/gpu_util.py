@@ -132,4 +132,6 @@ def run_small(wl, layer=0, key_depth=None, value_depth=None, prefix=None, block=
     torch.cuda.synchronize()
     assert_close(out.float().cpu().numpy(), ref_o, lse.cpu().numpy(), ref_l,
                  where=f"[{wl.name} layer {layer} kappa {kap} nu {nu}]")
+    # no wait ran out (attention pipeline or the merge's partial counters)
+    assert das.workspace_status(ws) & 1 == 0
     return out, lse, ws

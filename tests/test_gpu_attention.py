@@ -78,6 +78,46 @@ def test_weighted_split_threshold(P):
     run_small(small(batch=1, kv_heads=8, q_heads=8, prefix=(P, P), block=(8,)))
 
 
+def test_many_pairs():
+    """1600 (sequence, kv head) pairs over 152 CTAs, ragged lengths: ranges
+    that cross many pairs, a merge grid of thousands of CTAs."""
+    rng = np.random.default_rng(5)
+    B = 200
+    prefix = rng.integers(0, 200, size=B).astype(np.int32)
+    block = rng.integers(1, 5, size=B).astype(np.int32)
+    wl = small(batch=B, q_heads=8, kv_heads=8, head_dim=64, prefix=(0, 200), block=(4,))
+    run_small(wl, prefix=prefix, block=block)
+
+
+def test_one_workspace_across_shapes():
+    """A workspace sized for the largest of three shapes serves all of them in
+    turn, twice: nothing a call leaves in it but the status word affects the
+    next call, whatever its shape."""
+    import paper_2609_34538_gb300 as das
+    shapes = [small(batch=4, q_heads=16, kv_heads=8, prefix=(900, 3000), block=(8,)),
+              small(batch=1, q_heads=4, kv_heads=1, prefix=(20000, 20000), block=(16,)),
+              small(batch=2, q_heads=8, kv_heads=2, prefix=(5000, 5000), block=(4,))]
+    cases = []
+    for wl in shapes:
+        K, V = wl_mod.gen_cache(wl, depths=[2, 8])
+        P, T = wl.prefix_lens(), wl.block_lens()
+        q = wl_mod.gen_q(wl, 1)
+        kb, vb = wl_mod.gen_block_kv(wl, 1)
+        ref = oracle.attention(K, V, 1, 2, 8, P, T, q, kb, vb)
+        cache = das.DepthKVCache(dev_bf16(K), dev_bf16(V))
+        cases.append((wl, cache, dev_i32(P), dev_i32(T), dev_bf16(q), dev_bf16(kb), dev_bf16(vb), ref))
+    need = max(das.das_workspace_size(c[1], c[0].q_heads, c[0].max_block) for c in cases)
+    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    for rnd in range(2):
+        for wl, cache, pl, bl, q, kb, vb, (ro, rl) in cases:
+            n = das.das_workspace_size(cache, wl.q_heads, wl.max_block)
+            out, lse = das.das_mature_v_attention(cache, 1, 2, 8, pl, bl, q, kb, vb, ws[:n])
+            torch.cuda.synchronize()
+            assert_close(out.float().cpu().numpy(), ro, lse.cpu().numpy(), rl,
+                         where=f"[shared workspace, round {rnd}, B {wl.batch} Hkv {wl.kv_heads}]")
+            assert das.workspace_status(ws) == 0
+
+
 def test_sharp_softmax_scale():
     """scale = 1 makes the softmax peaked (the default 1/sqrt(D) is nearly flat here)."""
     run_small(small(q_heads=8, kv_heads=2, prefix=(500, 500), block=(8,)), scale=1.0)
