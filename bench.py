@@ -112,6 +112,32 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def graph_kernel_nodes(graph):
+    """Kernel nodes of a captured torch CUDA graph, read with the driver API
+    (cuGraphGetNodes, cuGraphNodeGetType); None if either is unavailable."""
+    import ctypes
+    raw = getattr(graph, "raw_cuda_graph", None)
+    if raw is None:
+        return None
+    try:
+        cu = ctypes.CDLL("libcuda.so.1")
+    except OSError:
+        return None
+    h = ctypes.c_void_p(raw())
+    n = ctypes.c_size_t(0)
+    if cu.cuGraphGetNodes(h, None, ctypes.byref(n)) != 0:
+        return None
+    nodes = (ctypes.c_void_p * max(1, n.value))()
+    if cu.cuGraphGetNodes(h, nodes, ctypes.byref(n)) != 0:
+        return None
+    kind, kernels = ctypes.c_int(0), 0
+    for i in range(n.value):
+        if cu.cuGraphNodeGetType(ctypes.c_void_p(nodes[i]), ctypes.byref(kind)) != 0:
+            return None
+        kernels += kind.value == 0  # CU_GRAPH_NODE_TYPE_KERNEL
+    return kernels
+
+
 def code_digest(path):
     """code_text_digest of a source file."""
     return code_text_digest(open(path, encoding="utf-8").read())
@@ -295,12 +321,26 @@ def gpu_arm(args):
         pl.copy_(P0)
         draft_phase(); verify_phase(); commit_phase()
     stream.synchronize()
-    graphs = []
+    # the library's launches per step: the kernel nodes of the three graphs
+    # (each holds library calls only), read before they are instantiated;
+    # the count of the launch sequence (L attention + L merge per attention
+    # phase, accept 1 or 2, append 2) if the graph cannot be read
+    graphs, nodes = [], []
     for fn in (draft_phase, verify_phase, commit_phase):
-        g = torch.cuda.CUDAGraph()
+        try:
+            g = torch.cuda.CUDAGraph(keep_graph=True)
+        except TypeError:
+            g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             fn()
+        try:
+            nodes.append(graph_kernel_nodes(g))
+        except RuntimeError:
+            nodes.append(None)
+        if hasattr(g, "instantiate"):
+            g.instantiate()
         graphs.append(g)
+    launches_per_step = (sum(nodes) if None not in nodes else None)
 
     def step(ev):
         with torch.cuda.stream(stream):
@@ -369,6 +409,8 @@ def gpu_arm(args):
                   for n in ("long", "decode", "batched", "verify") if n != args.workload}
         probes["long_2slab"] = draft_probe("long", dev, 200, 5, peak, compact=True)
         commit = commit_probe("verify", dev, 200, 5, peak)
+        # the single-sequence decode step's acceptance and commit ([1, 8, 32000])
+        commit["decode"] = commit_probe("decode", dev, 200, 5, peak, vocab=32000)
         del cache, K, V
         torch.cuda.empty_cache()
         seq, wave = decode_cache_probes(dev, 20, 3, peak)
@@ -427,7 +469,10 @@ def gpu_arm(args):
         "sequential_draft": seq,
         "das_wave_refinement": wave,
         "e4m3_cache_draft": f8,
-        "gpu_launches": K_steps * (2 * L * 2 + 2 + 2),
+        "gpu_launches": K_steps * (launches_per_step or (2 * L * 2 + 2 + 2)),
+        "gpu_launches_per_step": {"count": launches_per_step or (2 * L * 2 + 2 + 2),
+                                  "source": "kernel nodes of the step's CUDA graphs"
+                                  if launches_per_step else "launch sequence (two-kernel accept)"},
         "e2e": e2e,
         "cpu_baseline": cpu,
         "clocks": clocks.summary(),
@@ -516,7 +561,7 @@ def draft_probe(name, dev, steps, warmup, peak, layers=0, compact=False):
             "steps": len(ms)}
 
 
-def commit_probe(name, dev, steps, warmup, peak, layers=0, calls=4):
+def commit_probe(name, dev, steps, warmup, peak, layers=0, calls=4, vocab=0):
     """Greedy acceptance and the commit at a verify-and-commit workload's
     shape (Sec. 3.4, App. B.1), each timed on its own as a CUDA graph of
     `calls` back-to-back calls on distinct inputs (L2 flushed before every
@@ -536,6 +581,8 @@ def commit_probe(name, dev, steps, warmup, peak, layers=0, calls=4):
     wl = wlm.WORKLOADS[name]
     if layers:
         wl = wl.replace(layers=layers)
+    if vocab:  # a draft workload's commit: the logits of its block's rows
+        wl = wl.replace(vocab=vocab)
     W, B = wl.max_block, wl.batch
     wl = wl.replace(extra_capacity=(calls - 1) * W)
     stream = torch.cuda.Stream(device=dev)

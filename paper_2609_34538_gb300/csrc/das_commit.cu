@@ -16,20 +16,26 @@ namespace das {
 namespace {
 
 // ---- greedy acceptance and the DAS-Wave readout ------------------------------
-// Two steps, neither with scratch memory beyond the outputs:
-//   row_argmax_kernel: the first maximum of every logits row, row i of
-//     sequence b scanned by k CTAs (a cluster of k, each a 1/k slice of the
-//     vocabulary, k chosen so that rows * k fills the SMs, at most 8); CTA r
-//     of the cluster stores its best (value, index) straight into CTA 0's
-//     shared memory (distributed shared memory) and CTA 0 writes
-//       accept mode (Sec. 3.4):  target_ids[b][i];
-//       readout mode (Eq. 6, Sec. 3.3):  tokens[b][i + 1];
-//   accept_scan_kernel (accept mode only, a programmatic dependent of the
-//     first): one warp per sequence finds the first mismatch between
-//     draft_ids and target_ids and writes accepted and next_token.
+// No scratch memory beyond the outputs.  Greedy acceptance takes one of two
+// forms, chosen per launch:
+//   accept_fused_kernel (one kernel): a cluster of W * k CTAs is one
+//     sequence, row i scanned by CTAs i k .. i k + k - 1 (each a 1/k slice
+//     of the vocabulary); every CTA stores its best (value, index) straight
+//     into CTA 0's shared memory (distributed shared memory), and CTA 0
+//     writes target_ids[b][*], accepted[b] and next_token[b].  Used when
+//     W k <= 16 (k reduced to fit) and all B clusters are resident at once.
+//   row_argmax_kernel + accept_scan_kernel (two kernels): a cluster of k
+//     CTAs is one row, CTA 0 writes target_ids[b][i]; then one warp per
+//     sequence (a programmatic dependent) finds the first mismatch between
+//     draft_ids and target_ids and writes accepted and next_token.  It
+//     spreads rows over more SMs, and serves any B and W.
+// k is chosen so that rows * k fills the SMs (at most 8).  The DAS-Wave
+// readout (Eq. 6, Sec. 3.3) is row_argmax_kernel in readout mode, writing
+// tokens[b][i + 1].
 constexpr int kRowThreadsMax = 1024;
 constexpr int kRowLoads = 8;    // vector loads in flight per thread
 constexpr int kMaxRowCtas = 8;  // CTAs per row: a portable cluster
+constexpr int kMaxSeqCtas = 16; // CTAs of one sequence's cluster (a non-portable size)
 constexpr int kMaxW = 1024;
 constexpr int kScanWarps = 4;
 
@@ -58,33 +64,19 @@ struct RowArgs {
     int stride;
 };
 
-// VEC = 4: float4 loads (vocab % 4 == 0 and 16-byte aligned logits), else 1.
-// The cluster size k (1..8) is the launch's; row = blockIdx.x / k.
-template <int VEC, bool READOUT>
-__global__ void __launch_bounds__(kRowThreadsMax) row_argmax_kernel(const RowArgs a) {
-    __shared__ float warp_v[32];
-    __shared__ int warp_i[32];
-    __shared__ float cand_v[kMaxRowCtas];
-    __shared__ int cand_i[kMaxRowCtas];
-    cg::cluster_group cluster = cg::this_cluster();
-    const int k = (int)cluster.num_blocks();
-    const int rank = (int)cluster.block_rank();
-    const size_t row = blockIdx.x / k;
+// The first maximum (value, index) of logits src[lo, hi) over the whole CTA
+// (valid in thread 0): batches of kRowLoads vector loads per thread, all
+// issued before the compares, then warp and CTA reductions.  VEC = 4: float4
+// loads (vocab % 4 == 0 and 16-byte aligned logits, lo a multiple of 4), else 1.
+template <int VEC>
+__device__ __forceinline__ void slice_best(const float *__restrict__ row, int lo, int hi,
+                                           float &bv, int &bi, float *warp_v, int *warp_i) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // a CTA's shared memory may be written by another only once that CTA has
-    // started: every CTA arrives here and waits before its remote store
-    if (k > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
-    // the logits may come from the kernel before this one
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-
-    const int lo = min(rank * a.slice, a.vocab), hi = min(lo + a.slice, a.vocab);
-    const int nvec = (hi - lo) / VEC;  // slice is a multiple of VEC
-    const float *__restrict__ src = a.logits + row * (size_t)a.vocab + lo;
-    float bv = -INFINITY;
-    int bi = 0x7fffffff;
+    const int nvec = (hi - lo) / VEC;  // the slice is a multiple of VEC
+    const float *__restrict__ src = row + lo;
+    bv = -INFINITY;
+    bi = 0x7fffffff;
     const int nt = blockDim.x;
-    // batches of kRowLoads vector loads, all issued before the compares
     for (int j0 = threadIdx.x; j0 < nvec; j0 += kRowLoads * nt) {
         float x[kRowLoads][VEC];
 #pragma unroll
@@ -122,6 +114,30 @@ __global__ void __launch_bounds__(kRowThreadsMax) row_argmax_kernel(const RowArg
         bi = lane < (nt >> 5) ? warp_i[lane] : 0x7fffffff;
         warp_best(bv, bi);
     }
+}
+
+// The cluster size k (1..8) is the launch's; row = blockIdx.x / k.
+template <int VEC, bool READOUT>
+__global__ void __launch_bounds__(kRowThreadsMax) row_argmax_kernel(const RowArgs a) {
+    __shared__ float warp_v[32];
+    __shared__ int warp_i[32];
+    __shared__ float cand_v[kMaxRowCtas];
+    __shared__ int cand_i[kMaxRowCtas];
+    cg::cluster_group cluster = cg::this_cluster();
+    const int k = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const size_t row = blockIdx.x / k;
+    // a CTA's shared memory may be written by another only once that CTA has
+    // started: every CTA arrives here and waits before its remote store
+    if (k > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // the logits may come from the kernel before this one
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    const int lo = min(rank * a.slice, a.vocab), hi = min(lo + a.slice, a.vocab);
+    float bv;
+    int bi;
+    slice_best<VEC>(a.logits + row * (size_t)a.vocab, lo, hi, bv, bi, warp_v, warp_i);
     if (k > 1) {
         asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
         if (threadIdx.x == 0) {
@@ -147,6 +163,72 @@ __global__ void __launch_bounds__(kRowThreadsMax) row_argmax_kernel(const RowArg
             a.tokens[b * a.stride + i + 1] = t;
         } else {
             a.target_ids[row] = t;
+        }
+    }
+}
+
+// Greedy acceptance in one kernel.  The launch's cluster of n = W k CTAs
+// (n <= 16) is sequence b = blockIdx.x / n; CTA rank i k + r scans slice r
+// of row i.  CTA 0 gathers the n candidates, and its first warp (lane i for
+// row i) writes target_ids[b][i], then accepted[b] (the first mismatch with
+// draft_ids, by ballot) and next_token[b].
+template <int VEC>
+__global__ void __launch_bounds__(kRowThreadsMax)
+    accept_fused_kernel(const RowArgs a, const int32_t *__restrict__ draft,
+                        int32_t *__restrict__ accepted, int32_t *__restrict__ next_token) {
+    __shared__ float warp_v[32];
+    __shared__ int warp_i[32];
+    __shared__ float cand_v[kMaxSeqCtas];
+    __shared__ int cand_i[kMaxSeqCtas];
+    cg::cluster_group cluster = cg::this_cluster();
+    const int n = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int k = n / a.W;
+    const size_t b = blockIdx.x / n;
+    const int i = rank / k, r = rank % k;
+    if (n > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // the logits and draft ids may come from the kernel before this one
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    const int lo = min(r * a.slice, a.vocab), hi = min(lo + a.slice, a.vocab);
+    float bv;
+    int bi;
+    slice_best<VEC>(a.logits + (b * a.W + i) * (size_t)a.vocab, lo, hi, bv, bi, warp_v, warp_i);
+    if (n > 1) {
+        asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+        if (threadIdx.x == 0) {
+            *cluster.map_shared_rank(cand_v + rank, 0) = bv;
+            *cluster.map_shared_rank(cand_i + rank, 0) = bi;
+        }
+        // as in row_argmax_kernel: only CTA 0 waits and is read remotely
+        asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+        if (rank != 0) return;
+        asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+    } else if (threadIdx.x == 0) {
+        cand_v[0] = bv;
+        cand_i[0] = bi;
+    }
+    if (n == 1) __syncthreads();
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int32_t *d = draft + b * a.W;
+        int t = 0;
+        bool miss = false;
+        if (lane < a.W) {
+            float v = cand_v[lane * k];
+            int x = cand_i[lane * k];
+            for (int u = 1; u < k; ++u) better(v, x, cand_v[lane * k + u], cand_i[lane * k + u]);
+            t = x == 0x7fffffff ? 0 : x;  // a row of -inf: the first index
+            a.target_ids[b * a.W + lane] = t;
+            miss = d[lane] != t;
+        }
+        const unsigned m = __ballot_sync(0xffffffffu, miss);
+        const int first = m ? __ffs(m) - 1 : a.W;
+        const int t_first = __shfl_sync(0xffffffffu, t, first < a.W ? first : 0);
+        if (lane == 0) {
+            accepted[b] = first;
+            next_token[b] = first < a.W ? t_first : d[a.W - 1];
         }
     }
 }
@@ -343,6 +425,20 @@ cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, unsigne
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
 }
 
+// CTAs per row of the argmax step: k = SMs / rows clamped to [1, 8].
+int row_ctas(long long rows, int sms) {
+    return rows >= sms ? 1 : (int)std::min<long long>(kMaxRowCtas, sms / rows);
+}
+
+// Threads of an argmax CTA: enough for kRowLoads vector loads each over the
+// slice (a.slice must be set), a multiple of 32 in [32, 1024].
+template <int VEC>
+int row_threads(const RowArgs &a) {
+    const int nvec = a.slice / VEC;
+    const int t = (nvec + kRowLoads - 1) / kRowLoads;
+    return std::max(32, std::min(kRowThreadsMax, (t + 31) / 32 * 32));
+}
+
 // The argmax step: k CTAs per row, k = SMs / rows clamped to [1, 8], with
 // enough threads for kRowLoads vector loads each over a 1/k slice.
 template <int VEC, bool READOUT>
@@ -352,15 +448,12 @@ cudaError_t row_argmax_launch(RowArgs a, long long rows, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     const int sms = attn_grid_size(dev);
     if (sms <= 0) return cudaErrorInvalidDevice;
-    const int k = rows >= sms ? 1 : (int)std::min<long long>(kMaxRowCtas, sms / rows);
+    const int k = row_ctas(rows, sms);
     const int slice = (a.vocab + k - 1) / k;
     a.slice = (slice + VEC - 1) / VEC * VEC;
-    const int nvec = a.slice / VEC;
-    int threads = (nvec + kRowLoads - 1) / kRowLoads;
-    threads = std::max(32, std::min(kRowThreadsMax, (threads + 31) / 32 * 32));
     if (rows * k > 0x7fffffffLL) return cudaErrorInvalidValue;
     return launch_pdl(row_argmax_kernel<VEC, READOUT>, dim3((unsigned)(rows * k)),
-                      dim3((unsigned)threads), (unsigned)k, stream, a);
+                      dim3((unsigned)row_threads<VEC>(a)), (unsigned)k, stream, a);
 }
 
 cudaError_t argmax_launch(const RowArgs &a, int B, bool readout, cudaStream_t stream) {
@@ -375,18 +468,92 @@ cudaError_t argmax_launch(const RowArgs &a, int B, bool readout, cudaStream_t st
                : row_argmax_launch<1, false>(a, rows, stream);
 }
 
+// Clusters of n CTAs of kRowThreadsMax threads (an upper bound on the
+// launch's) that can be resident at once, looked up once per device and n.
+template <int VEC>
+cudaError_t fused_resident_clusters(int dev, int n, int &clusters) {
+    static std::atomic<int> cached[64][kMaxSeqCtas + 1];
+    if (dev < 64) {
+        const int c = cached[dev][n].load(std::memory_order_relaxed);
+        if (c > 0) {
+            clusters = c - 1;
+            return cudaSuccess;
+        }
+    }
+    cudaError_t e = cudaFuncSetAttribute(accept_fused_kernel<VEC>,
+                                         cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)n);
+    cfg.blockDim = dim3(kRowThreadsMax);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)n;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaOccupancyMaxActiveClusters(&clusters, accept_fused_kernel<VEC>, &cfg);
+    if (e != cudaSuccess) return e;
+    if (dev < 64) cached[dev][n].store(clusters + 1, std::memory_order_relaxed);
+    return cudaSuccess;
+}
+
+// k > 0: greedy acceptance runs as accept_fused_kernel with k CTAs per row
+// (the two-kernel form's k, or fewer so that W k <= 16) when every
+// sequence's cluster of W k CTAs is resident at once (one wave); otherwise
+// k = 0 (the two-kernel form).  On a 152-SM GB300 at most 7 clusters of 16
+// CTAs (15 of 8) are resident, so [8, 16, vocab] stays two-kernel, while a
+// single sequence's accept (B 1, W 8) gains the second kernel's dependency
+// wait: 6.18 -> 5.02 us over a 32000 vocabulary (B 2 to 4 at W 16: equal).
+cudaError_t fused_accept_ctas(int B, int W, bool vec, int &k) {
+    k = 0;
+    if (W > kMaxSeqCtas) return cudaSuccess;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const int sms = attn_grid_size(dev);
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    const int kr = std::min(row_ctas((long long)B * W, sms), kMaxSeqCtas / W);
+    int clusters = 0;
+    e = vec ? fused_resident_clusters<4>(dev, W * kr, clusters)
+            : fused_resident_clusters<1>(dev, W * kr, clusters);
+    if (e != cudaSuccess) return e;
+    if (B <= clusters) k = kr;
+    return cudaSuccess;
+}
+
+template <int VEC>
+cudaError_t accept_fused_launch(RowArgs a, int B, int k, const int32_t *draft,
+                                int32_t *accepted, int32_t *next_token, cudaStream_t stream) {
+    const int slice = (a.vocab + k - 1) / k;
+    a.slice = (slice + VEC - 1) / VEC * VEC;
+    const int n = a.W * k;
+    return launch_pdl(accept_fused_kernel<VEC>, dim3((unsigned)(B * n)),
+                      dim3((unsigned)row_threads<VEC>(a)), (unsigned)n, stream, a, draft,
+                      accepted, next_token);
+}
+
 }  // namespace
 
 cudaError_t accept_launch(const float *logits, const int32_t *draft, int B, int W, int vocab,
                           int32_t *accepted, int32_t *target_ids, int32_t *next_token,
                           cudaStream_t stream) {
+    if (B == 0) return cudaSuccess;
     RowArgs a = {};
     a.logits = logits;
     a.W = W;
     a.vocab = vocab;
     a.target_ids = target_ids;
-    cudaError_t e = argmax_launch(a, B, false, stream);
-    if (e != cudaSuccess || B == 0) return e;
+    const bool vec = (vocab % 4) == 0 && (reinterpret_cast<uintptr_t>(logits) & 15u) == 0;
+    int k = 0;
+    cudaError_t e = fused_accept_ctas(B, W, vec, k);
+    if (e != cudaSuccess) return e;
+    if (k > 0)
+        return vec ? accept_fused_launch<4>(a, B, k, draft, accepted, next_token, stream)
+                   : accept_fused_launch<1>(a, B, k, draft, accepted, next_token, stream);
+    e = argmax_launch(a, B, false, stream);
+    if (e != cudaSuccess) return e;
     return launch_pdl(accept_scan_kernel, dim3((unsigned)((B + kScanWarps - 1) / kScanWarps)),
                       dim3(kScanWarps * 32), 1, stream, static_cast<const int32_t *>(target_ids),
                       draft, B, W, accepted, next_token);

@@ -41,6 +41,44 @@ def test_accept_shapes(B, W, V):
     check_accept(logits, draft)
 
 
+@pytest.mark.parametrize("B,W,V", [(1, 8, 32000), (2, 16, 32000), (7, 16, 32000), (3, 4, 4099),
+                                   (6, 5, 50257), (1, 1, 32000), (100, 1, 4096), (4, 3, 131072),
+                                   (8, 16, 32000), (16, 8, 32000)])
+def test_accept_single_kernel_shapes(B, W, V):
+    """Shapes whose sequences fit one cluster of W k <= 16 CTAs (k CTAs per
+    row).  They run as one kernel when the device holds all B clusters at
+    once, else as the two-kernel form: on a 152-SM GB300 (7 resident clusters
+    of 16 CTAs, 15 of 8) all but the last two run as one kernel, with k = 2,
+    1, 1, 4, 3, 8, 1 and 5.  Bit-exact either way, planted acceptance
+    lengths 0..W."""
+    a_star, draft, logits = synth.accept_inputs(B * 1000 + W, B, W, V)
+    acc, _, _ = check_accept(logits, draft)
+    assert np.array_equal(acc, a_star)
+
+
+@pytest.mark.parametrize("B,W", [(1, 1), (1, 2), (2, 4), (6, 5), (1, 8), (8, 16)])
+@pytest.mark.parametrize("V", [4099, 4096])
+def test_accept_ties_at_every_split(B, W, V):
+    """Every row holds its maximum on both sides of the slice boundary of
+    every k-way split, k = 2..8 (slices of ceil(V / k) columns, rounded up to
+    whole float4s when V % 4 == 0): whatever k either form of the kernel
+    picks, equal maxima sit in several CTAs' slices, and the smallest index
+    (the left side of the 8-way boundary) must win."""
+    logits = np.zeros((B, W, V), dtype=np.float32)
+    cols = []
+    for k in range(2, 9):
+        sl = -(-V // k)
+        if V % 4 == 0:
+            sl = -(-sl // 4) * 4
+        cols += [sl - 1, sl]
+    logits[:, :, cols] = 7.0
+    first = min(cols)
+    draft = np.full((B, W), first, dtype=np.int32)
+    draft[:, W - 1] = first + 1  # the last proposal is rejected
+    acc, tid, nxt = check_accept(logits, draft)
+    assert np.all(tid == first) and np.all(acc == W - 1) and np.all(nxt == first)
+
+
 def test_accept_ties_and_infinities():
     """Equal maxima go to the smallest index; rows of -inf give index 0."""
     B, W, V = 3, 4, 4099
@@ -56,16 +94,18 @@ def test_accept_ties_and_infinities():
     assert list(acc) == [4, 3, 3]
 
 
-@pytest.mark.parametrize("B", [1, 8, 32])
+@pytest.mark.parametrize("B,W", [(1, 7), (8, 7), (32, 7), (2, 4), (6, 5)])
 @pytest.mark.parametrize("V", [4099, 4096])
-def test_accept_ties_across_slices(B, V):
+def test_accept_ties_across_slices(B, W, V):
     """Equal maxima on both sides of a boundary between two CTAs' vocabulary
-    slices: a row is scanned by k CTAs (k = SMs / rows, 1..8; slices of
-    ceil(V / k) columns, rounded up to whole float4s when V % 4 == 0).  Row
-    k - 2 of every sequence holds a tie straddling the boundary of a k-way
-    split, so whatever k the launch picks, some row's tie crosses CTAs; the
-    smaller index wins either way."""
-    W = 7
+    slices: a row is scanned by k CTAs (k = SMs / rows, 1..8, or fewer in
+    the one-kernel form; slices of ceil(V / k) columns, rounded up to whole
+    float4s when V % 4 == 0).  Row r of every sequence holds a tie
+    straddling the boundary of an (r + 2)-way split, so whatever k the
+    launch picks (up to W + 1), some row's tie crosses CTAs; the smaller
+    index wins either way.  On a 152-SM GB300: B 1 W 7, B 2 W 4 and B 6 W 5
+    run as one kernel with k = 2, 4 and 3; B 8 and 32 at W 7 as two kernels
+    with k = 2 and 1."""
     logits = np.zeros((B, W, V), dtype=np.float32)
     draft = np.zeros((B, W), dtype=np.int32)
     first = []
