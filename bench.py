@@ -581,8 +581,8 @@ def commit_probe(name, dev, steps, warmup, peak, layers=0, calls=4, vocab=0):
     wl = wlm.WORKLOADS[name]
     if layers:
         wl = wl.replace(layers=layers)
-    if vocab:  # a draft workload's commit: the logits of its block's rows
-        wl = wl.replace(vocab=vocab)
+    if vocab or not wl.vocab:  # a draft workload's commit: logits of its block's rows
+        wl = wl.replace(vocab=vocab or 32000)
     W, B = wl.max_block, wl.batch
     wl = wl.replace(extra_capacity=(calls - 1) * W)
     stream = torch.cuda.Stream(device=dev)

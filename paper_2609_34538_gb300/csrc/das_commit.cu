@@ -518,7 +518,10 @@ cudaError_t fused_accept_ctas(int B, int W, bool vec, int &k) {
     int clusters = 0;
     e = vec ? fused_resident_clusters<4>(dev, W * kr, clusters)
             : fused_resident_clusters<1>(dev, W * kr, clusters);
-    if (e != cudaSuccess) return e;
+    if (e != cudaSuccess) {  // a device without that cluster size: the two-kernel form
+        (void)cudaGetLastError();
+        return cudaSuccess;
+    }
     if (B <= clusters) k = kr;
     return cudaSuccess;
 }
