@@ -270,10 +270,15 @@ size_t das_workspace_size_f8(const das_kv_cache_f8 *cache, int num_q_heads, int 
 /*
  * das_mature_v_attention over a das_kv_cache_f8: keys are read at key_depth
  * and values at value_depth from k_top / v_top (depth R) or from k_low / v_low
- * (depths below R, e4m3, widened exactly to bf16 before the products), so
- * Eqs. 2-3 are evaluated on the stored values.  key_depth = value_depth = d
- * is the verify attention of depth d (Sec. 3.4).  All other arguments,
- * results and limits as das_mature_v_attention.
+ * (depths below R, e4m3), so Eqs. 2-3 are evaluated on the stored values.
+ * key_depth = value_depth = d is the verify attention of depth d (Sec. 3.4).
+ * All other arguments, results and limits as das_mature_v_attention.
+ * e4m3 operands are widened exactly to bf16 before the products, except for
+ * e4m3 keys with bf16 values at head_dim 128 (Mature-V, key_depth < R =
+ * value_depth): there the scores are e4m3 products of the stored keys with
+ * each query row split exactly into two e4m3 parts under a power of two per
+ * row (exact for elements down to about 2^-9 of the row's largest magnitude,
+ * fp32 accumulation), and the queries must be finite.
  */
 das_status das_mature_v_attention_f8(const das_kv_cache_f8 *cache, int layer, int key_depth,
                                      int value_depth, const int32_t *prefix_len,

@@ -31,9 +31,10 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 // Tensor map over `rank` dims (innermost first): bf16 elements with 128-byte
 // swizzle, or 8-bit (e4m3) elements without swizzle (their tiles are widened
-// by the kernel, which reads them row by row).
+// by the kernel, which reads them row by row) or, with swizzle8, with 128-byte
+// swizzle (key tiles of 128-byte rows that the e4m3 MMAs read as they land).
 bool encode_uncached(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
-                     const cuuint32_t *box, bool e4m3) {
+                     const cuuint32_t *box, bool e4m3, bool swizzle8) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t strides[4];
@@ -52,7 +53,7 @@ bool encode_uncached(CUtensorMap *m, void *base, int rank, const cuuint64_t *dim
                                                             : CU_TENSOR_MAP_L2_PROMOTION_L2_64B;
     return fn(m, e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
               (cuuint32_t)rank, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-              e4m3 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B, promo,
+              e4m3 && !swizzle8 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B, promo,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -64,7 +65,7 @@ bool encode_uncached(CUtensorMap *m, void *base, int rank, const cuuint64_t *dim
 struct MapKey {
     void *base;
     int rank;
-    bool e4m3;
+    bool e4m3, swizzle8;
     cuuint64_t dims[5];
     cuuint32_t box[5];
 };
@@ -78,18 +79,20 @@ std::mutex g_map_mu;
 MapSlot g_maps[kMapSlots];
 
 bool same_key(const MapKey &a, const MapKey &b) {
-    if (a.base != b.base || a.rank != b.rank || a.e4m3 != b.e4m3) return false;
+    if (a.base != b.base || a.rank != b.rank || a.e4m3 != b.e4m3 || a.swizzle8 != b.swizzle8)
+        return false;
     for (int i = 0; i < a.rank; ++i)
         if (a.dims[i] != b.dims[i] || a.box[i] != b.box[i]) return false;
     return true;
 }
 
 bool encode(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
-            const cuuint32_t *box_in, bool e4m3) {
+            const cuuint32_t *box_in, bool e4m3, bool swizzle8 = false) {
     MapKey key = {};
     key.base = base;
     key.rank = rank;
     key.e4m3 = e4m3;
+    key.swizzle8 = swizzle8;
     const cuuint32_t box_default[5] = {64, 1, 64, 1, 1};
     for (int i = 0; i < rank; ++i) {
         key.dims[i] = dims[i];
@@ -103,7 +106,7 @@ bool encode(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
         }
     };
     mix(reinterpret_cast<uintptr_t>(base));
-    mix((uint64_t)rank * 2 + (e4m3 ? 1 : 0));
+    mix((uint64_t)rank * 4 + (e4m3 ? 1 : 0) + (swizzle8 ? 2 : 0));
     for (int i = 0; i < rank; ++i) {
         mix(key.dims[i]);
         mix(key.box[i]);
@@ -116,7 +119,7 @@ bool encode(CUtensorMap *m, void *base, int rank, const cuuint64_t *dims,
             return true;
         }
     }
-    if (!encode_uncached(m, base, rank, key.dims, key.box, e4m3)) return false;
+    if (!encode_uncached(m, base, rank, key.dims, key.box, e4m3, swizzle8)) return false;
     std::lock_guard<std::mutex> lock(g_map_mu);
     slot.used = true;
     slot.key = key;
@@ -180,16 +183,19 @@ das_status attention_core(const Shape &c, int layer, Operand key, Operand value,
 
     const int D = c.head_dim;
     CUtensorMap tk, tv, tkb, tvb, tq;
-    auto operand_map = [&](CUtensorMap *m, const Operand &o) {
+    auto operand_map = [&](CUtensorMap *m, const Operand &o, bool swizzle8) {
         const cuuint64_t dims[5] = {(cuuint64_t)D, (cuuint64_t)c.kv_heads, (cuuint64_t)c.capacity,
                                     (cuuint64_t)c.batch, (cuuint64_t)o.slabs};
         // e4m3: one {D, 1, 64} box per tile; bf16: {64, 1, 64} swizzled panels
         const cuuint32_t box8[5] = {(cuuint32_t)D, 1, 64, 1, 1};
-        return encode(m, o.base, 5, dims, o.e4m3 ? box8 : nullptr, o.e4m3);
+        return encode(m, o.base, 5, dims, o.e4m3 ? box8 : nullptr, o.e4m3, swizzle8);
     };
+    // e4m3 keys with bf16 values at D = 128 are read by the e4m3 MMAs straight
+    // from the 128-byte-swizzled tile (the kernel's query-split path)
+    const bool key_swizzle8 = key.e4m3 && !value.e4m3 && D == 128;
     const cuuint64_t blk_dims[4] = {(cuuint64_t)D, (cuuint64_t)c.kv_heads, (cuuint64_t)max_block,
                                     (cuuint64_t)c.batch};
-    if (!operand_map(&tk, key) || !operand_map(&tv, value) ||
+    if (!operand_map(&tk, key, key_swizzle8) || !operand_map(&tv, value, false) ||
         !encode_bf16(&tkb, const_cast<void *>(k_blk), 4, blk_dims) ||
         !encode_bf16(&tvb, const_cast<void *>(v_blk), 4, blk_dims))
         return DAS_ERR_CUDA;

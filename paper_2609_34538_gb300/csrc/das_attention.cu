@@ -72,7 +72,8 @@ constexpr int kSBufs = 4;            // S buffers in tensor memory
 constexpr int kPrefetchTiles = 2;    // prefix tiles pulled into L2 before the dependency wait
 constexpr int kLongRange = 80;       // ranges longer than this prefetch one tile (measured:
                                      // long / verify 0.45 us faster, decode and batched not)
-constexpr int kTmemCols = 512;       // S buffers [0, 64 kSBufs), O [64 kSBufs, 64 kSBufs + D)
+constexpr int kTmemCols = 512;       // S buffers [0, 64 kSBufs), O [64 kSBufs, 64 kSBufs + D),
+                                     // then 8 columns whose first is the rounded row sum
 constexpr float kRescaleLog2 = 8.f;  // move the reference max only beyond 2^8
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -187,6 +188,18 @@ __device__ __forceinline__ void mma(uint32_t d_tmem, uint64_t a, uint64_t b, uin
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
         " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(id), "r"(accumulate)
+        : "memory");
+}
+// kind::f8f6f4 with e4m3 A and B (format code 0 for both), fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_e4m3(int M, int N) {
+    return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(id), "r"(accumulate)
         : "memory");
 }
@@ -525,18 +538,26 @@ __device__ bool plan(const AttnParams &p, int P0, int T0, long long &lo, long lo
 }
 
 // Shared memory of one CTA.  Keys and values stored as e4m3 (the depths below
-// R in a das_kv_cache_f8) land in the stage as 8-bit tiles [64 keys][D] and
-// are widened by the conversion warps into bf16 tiles, in the
-// 128-byte-swizzled layout the MMAs read, held in a ring of kConvSlots slots
-// (tile j in slot j % kConvSlots) rather than one per stage: the smaller
-// stages then fit 6 (or 7) deep instead of 4, which is what keeps more DRAM
-// requests in flight per SM.  A pair's block tile is bf16: the conversion
-// warps load its e4m3-stored operands straight into the ring slot, the
-// producer the others into the stage.
+// R in a das_kv_cache_f8) land in the stage as 8-bit tiles [64 keys][D].
+//   kQSplit (keys e4m3, values bf16, D = 128: Mature-V over a das_kv_cache_f8):
+//     the key tile lands 128-byte swizzled and is read by the S MMAs as it is
+//     (kind::f8f6f4).  The conversion warps split each segment's bf16 query
+//     rows exactly into two e4m3 parts, 2^e q = hi + lo with one power of two
+//     e per row (see split_q), and S = (hi + lo) K^T is two e4m3 products
+//     accumulated in fp32, 2^e times the bf16 product.  The pair's block
+//     tile (bf16 keys) has a bf16 key buffer of its own and bf16 MMAs.
+//   otherwise: the conversion warps widen every e4m3 tile into bf16 tiles, in
+//     the 128-byte-swizzled layout the MMAs read, held in a ring of kConvSlots
+//     slots (tile j in slot j % kConvSlots) rather than one per stage: the
+//     smaller stages then fit 6 (or 7) deep instead of 4, which is what keeps
+//     more DRAM requests in flight per SM.  A pair's block tile is bf16: the
+//     conversion warps load its e4m3-stored operands straight into the ring
+//     slot, the producer the others into the stage.
 template <int D, bool KF8, bool VF8>
 struct Layout {
+    static constexpr bool kQSplit = KF8 && !VF8 && D == 128;
     static constexpr bool kConv = KF8 || VF8;
-    static constexpr int kStages = (KF8 && VF8) ? 7 : kConv ? 6 : 4;
+    static constexpr int kStages = kQSplit ? 5 : (KF8 && VF8) ? 7 : kConv ? 6 : 4;
     static constexpr int kConvSlots = 2;
     static constexpr int kThreads = (kSoftWarps + 3 + (kConv ? kConvWarps : 0)) * 32;
     static constexpr int kPanels = D / 64;
@@ -545,21 +566,31 @@ struct Layout {
     static constexpr int kKBytes = KF8 ? kTile8Bytes : kTileBytes;  // K part of a stage
     static constexpr int kVBytes = VF8 ? kTile8Bytes : kTileBytes;  // V part of a stage
     static constexpr int kStageBytes = kKBytes + kVBytes;
-    static constexpr int kConvBytes = (KF8 ? kTileBytes : 0) + (VF8 ? kTileBytes : 0);
+    static constexpr int kConvBytes =
+        kQSplit ? 0 : (KF8 ? kTileBytes : 0) + (VF8 ? kTileBytes : 0);
     static constexpr int kQBytes = kPanels * kRows * 128;  // one query buffer
+    static constexpr int kQ8Bytes = kRows * 128;           // one e4m3 query part (D = 128)
     static constexpr int kPBytes = kRows * kTileKeys * 2;  // one P buffer
     static constexpr int kStagesOff = 0;
-    static constexpr int kConvOff = kStages * kStageBytes;  // the ring of widened tiles
-    static constexpr int kQOff = kConvOff + kConvSlots * kConvBytes;
+    static constexpr int kConvOff = kStages * kStageBytes;  // the ring of widened tiles, or
+    // (kQSplit) the block tile's bf16 keys, then hi / lo of both query buffers
+    static constexpr int kBlkKOff = kConvOff;
+    static constexpr int kQ8Off = kConvOff + kTileBytes;
+    static constexpr int kExtraBytes =
+        kQSplit ? kTileBytes + 4 * kQ8Bytes : kConvSlots * kConvBytes;
+    static constexpr int kQOff = kConvOff + kExtraBytes;
     static constexpr int kPOff = kQOff + 2 * kQBytes;
-    static constexpr int kBarOff = kPOff + 2 * kPBytes;
+    // the B operand of the row-sum MMA: [8][64] bf16, row 0 ones, 128-byte swizzled
+    static constexpr int kOnesOff = kPOff + 2 * kPBytes;
+    static constexpr int kBarOff = kOnesOff + 1024;
     // barriers: full[kStages], empty[kStages], qfull[2], qempty[2],
     // sready[kSBufs], sfree[kSBufs], pready[2], pvdone[2], drain[2],
-    // cready[kConvSlots], kfree[kConvSlots], vfree[kConvSlots]
-    static constexpr int kNumBars = 2 * kStages + 10 + 2 * kSBufs + 3 * kConvSlots;
+    // cready[kConvSlots], kfree[kConvSlots], vfree[kConvSlots], qsplit[2], bkfree
+    static constexpr int kNumBars = 2 * kStages + 10 + 2 * kSBufs + 3 * kConvSlots + 3;
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kLenOff = kMiscOff + 16;  // lengths read before the dependency wait
-    static constexpr int kBytes = kLenOff + 64 * 4 + 1024;  // + alignment slack
+    static constexpr int kQeOff = kLenOff + 64 * 4;  // (kQSplit) e of each row, per query buffer
+    static constexpr int kBytes = kQeOff + (kQSplit ? 2 * kRows * 4 : 0) + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
     static_assert(kBytes <= 232448, "shared memory per CTA");
@@ -628,10 +659,91 @@ __device__ __forceinline__ void widen_tile(uint32_t src, uint32_t dst, int ct) {
     }
 }
 
+// Exact split of the query rows for e4m3 keys (D = 128).  Row r of the bf16
+// query buffer q (two 128-byte-swizzled panels of [64 rows][64 dims]) becomes
+// two e4m3 rows hi, lo (128-byte swizzled [64 rows][128 dims]) with
+//   2^e q = hi + lo,  e = 7 - floor(log2 max_d |q_d|)  (clamped to +-120),
+// so that the row's largest element scales into [128, 256).  hi is 2^e q
+// rounded to e4m3 (4 significant bits) and lo the rounded remainder: a bf16
+// value has 8 significant bits, so the remainder fits e4m3 exactly unless it
+// falls below e4m3's smallest subnormal (2^-9), i.e. for elements below about
+// 2^-9 of the row's largest.  Thread ct of the 128 conversion threads takes
+// row ct / 2, dims [64 (ct % 2), +64); e is written to qexp[row].  A row of
+// zeros gives e = 0; the query must be finite.
+__device__ __forceinline__ void split_q(uint32_t q, uint32_t hi, uint32_t lo, int *qexp, int ct) {
+    const int row = ct >> 1, half = ct & 1;
+    uint32_t w[32];
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(w[4 * c]), "=r"(w[4 * c + 1]), "=r"(w[4 * c + 2]), "=r"(w[4 * c + 3])
+                     : "r"(q + half * (kRows * 128) + row * 128 + ((c ^ (row & 7)) << 4)));
+    float mx = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        mx = fmaxf(mx, fmaxf(fabsf(__uint_as_float(w[i] << 16)),
+                             fabsf(__uint_as_float(w[i] & 0xffff0000u))));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    int e = 0;
+    if (mx > 0.f && mx <= 3.4e38f) {
+        e = 7 - ((int)((__float_as_uint(mx) >> 23) & 0xffu) - 127);
+        e = e < -120 ? -120 : (e > 120 ? 120 : e);
+    }
+    const float sc = __uint_as_float((uint32_t)(127 + e) << 23);
+    // word i holds dims 2i (low half) and 2i + 1 of the thread's 64
+    uint32_t h[16], l[16];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        const float xa = __uint_as_float(w[i] << 16) * sc;
+        const float xb = __uint_as_float(w[i] & 0xffff0000u) * sc;
+        uint32_t h2, f2, l2;
+        asm("{\n .reg .b16 t;\n cvt.rn.satfinite.e4m3x2.f32 t, %1, %2;\n cvt.u32.u16 %0, t;\n}"
+            : "=r"(h2)
+            : "f"(xb), "f"(xa));
+        asm("{\n .reg .b16 t;\n cvt.u16.u32 t, %1;\n cvt.rn.f16x2.e4m3x2 %0, t;\n}"
+            : "=r"(f2)
+            : "r"(h2));
+        float ha, hb;
+        asm("{\n .reg .b16 a, b;\n mov.b32 {a, b}, %2;\n cvt.f32.f16 %0, a;\n cvt.f32.f16 %1, b;\n}"
+            : "=f"(ha), "=f"(hb)
+            : "r"(f2));
+        asm("{\n .reg .b16 t;\n cvt.rn.satfinite.e4m3x2.f32 t, %1, %2;\n cvt.u32.u16 %0, t;\n}"
+            : "=r"(l2)
+            : "f"(xb - hb), "f"(xa - ha));
+        if (i & 1) {
+            h[i >> 1] |= h2 << 16;
+            l[i >> 1] |= l2 << 16;
+        } else {
+            h[i >> 1] = h2;
+            l[i >> 1] = l2;
+        }
+    }
+    // 16-byte chunk c of the 128-byte e4m3 row holds dims 16 c .. 16 c + 15:
+    // this thread's are chunks 4 half .. 4 half + 3
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+        const uint32_t off = row * 128 + (((4 * half + m) ^ (row & 7)) << 4);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(hi + off), "r"(h[4 * m]),
+                     "r"(h[4 * m + 1]), "r"(h[4 * m + 2]), "r"(h[4 * m + 3])
+                     : "memory");
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(lo + off), "r"(l[4 * m]),
+                     "r"(l[4 * m + 1]), "r"(l[4 * m + 2]), "r"(l[4 * m + 3])
+                     : "memory");
+    }
+    if (half == 0) qexp[row] = e;
+}
+
+// Registers a thread of the query-split variant may use: 144 x 352 threads
+// leave room for one merge CTA (128 threads x 116) beside the attention CTA,
+// so the merge kernel is resident before the attention grid ends (measured:
+// the e4m3 long call 89.9 -> 89.0 us against 165 registers, no spills).
+template <int D, bool KF8, bool VF8>
+constexpr int kRegCap = Layout<D, KF8, VF8>::kQSplit ? 144 : 255;
+
 // KF8 / VF8: prefix keys / values are e4m3 (tm_k / tm_v are 8-bit maps).
 template <int D, bool KF8, bool VF8>
 __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
-    attn_kernel(const __grid_constant__ CUtensorMap tm_k,
+    __maxnreg__((kRegCap<D, KF8, VF8>)) attn_kernel(const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_kb,
                    const __grid_constant__ CUtensorMap tm_vb,
@@ -648,8 +760,11 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                    b_sfree = b_sready + 8 * kSBufs, b_pready = b_sfree + 8 * kSBufs,
                    b_pvdone = b_pready + 16, b_drain = b_pvdone + 16,
                    b_cready = b_drain + 16, b_kfree = b_cready + 8 * Lt::kConvSlots,
-                   b_vfree = b_kfree + 8 * Lt::kConvSlots;
+                   b_vfree = b_kfree + 8 * Lt::kConvSlots,
+                   b_qsplit = b_vfree + 8 * Lt::kConvSlots, b_bkfree = b_qsplit + 16;
     constexpr int kSlots = Lt::kConvSlots;
+    constexpr bool kQSplit = Lt::kQSplit;
+    int *qexp = reinterpret_cast<int *>(sm + Lt::kQeOff);  // [2][kRows]
     // where the MMAs read tile j's bf16 K and V (stage s = j % kStages): the
     // TMA tile in the stage, or the ring slot j % kSlots the conversion warps
     // widened it into
@@ -685,9 +800,13 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(b_qfull + 8 * i, 1);
-            mbar_init(b_qempty + 8 * i, 1);
+            // kQSplit: the last S of the segment and every softmax warp, once
+            // it has read its row's e (the next split overwrites it)
+            mbar_init(b_qempty + 8 * i, kQSplit ? 1 + kSoftWarps : 1);
             mbar_init(b_pready + 8 * i, kSoftWarps);
+            mbar_init(b_qsplit + 8 * i, kConvWarps);
         }
+        mbar_init(b_bkfree, 1);
         for (int i = 0; i < kSBufs; ++i) {
             mbar_init(b_sready + 8 * i, 1);
             mbar_init(b_sfree + 8 * i, kSoftWarps);
@@ -725,6 +844,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     if (spec && warp == kProducerWarp) {
         len_sm[lane0] = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
         len_sm[32 + lane0] = lane0 < p.B ? len_cg(p.block_len, lane0, p.max_block) : 0;
+    }
+    if (threadIdx.x < 64) {  // the row-sum MMA's B operand: row 0 of [8][64] bf16 ones
+        const uint32_t one2 = threadIdx.x < 8 ? 0x3F803F80u : 0u;
+        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                         sbase + Lt::kOnesOff + threadIdx.x * 16),
+                     "r"(one2)
+                     : "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     if (warp == kProducerWarp && elect_one()) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
@@ -775,6 +902,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     // first steps may run before the lengths are checked (below).
     Walk wl = w0;
     int qseg = -1;
+    long long nblk = 0;           // (kQSplit) block tiles whose keys were issued
     long long issued = 0, j = 0;  // tiles whose loads were issued; next tile
     bool ok = true;
     uint64_t policy = 0;
@@ -801,6 +929,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         if (j >= kStages)
             ok = ok && wait(b_empty + 8 * s, (uint32_t)(((j - kStages) / kStages) & 1),
                             abort_flag, p.status);
+        const bool blk = wl.t == wl.nt - 1;
+        // (kQSplit) the block-key buffer is free once the S of the last block tile is done
+        if (kQSplit && blk && nblk >= 1)
+            ok = ok && wait(b_bkfree, (uint32_t)((nblk - 1) & 1), abort_flag, p.status);
         if (ok && elect_one()) {
             const uint32_t full = b_full + 8 * s;
             const uint32_t kdst = sbase + Lt::kStagesOff + s * Lt::kStageBytes;
@@ -825,6 +957,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                         tma_5d(vdst + dp * 8192, &tm_v, full, dp * 64, wl.h, tok, wl.b,
                                p.value_slab, policy);
                 }
+            } else if (kQSplit) {  // the block's own K (bf16) into its buffer, V into the stage
+                mbar_arrive_expect_tx(full, 2 * Lt::kTileBytes);
+#pragma unroll
+                for (int dp = 0; dp < Lt::kPanels; ++dp) {
+                    tma_4d(sbase + Lt::kBlkKOff + dp * 8192, &tm_kb, full, dp * 64, wl.h, 0,
+                           wl.b);
+                    tma_4d(vdst + dp * 8192, &tm_vb, full, dp * 64, wl.h, 0, wl.b);
+                }
             } else {  // the block's own K / V (bf16): the operands read from the
                       // stage; ring-slot operands are loaded by the conversion warps
                 mbar_arrive_expect_tx(full, (KF8 ? 0 : Lt::kTileBytes) +
@@ -837,6 +977,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             }
         }
         __syncwarp();
+        if (ok && kQSplit && blk) ++nblk;
         if (ok) issued = j + 1;
         walk_next(p, wl);
         ++j;
@@ -848,7 +989,8 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
     // the first loads of the speculative plan go out while the lengths are
     // checked (no step here waits: fresh stages and query buffers only)
     if (spec && warp == kProducerWarp)
-        while (j < ntiles && j < kStages && ok && !((j == 0 || wl.t == 0) && qseg + 1 >= 2))
+        while (j < ntiles && j < kStages && ok && !((j == 0 || wl.t == 0) && qseg + 1 >= 2) &&
+               !(kQSplit && wl.t == wl.nt - 1 && nblk >= 1))
             produce();
     {
         const int P1 = lane0 < p.B ? len_cg(p.prefix_len, lane0, p.capacity) : 0;
@@ -869,6 +1011,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             ntiles = plan(p, P1, T1, lo, hi, w0) ? hi - lo : 0;
             wl = w0;
             qseg = -1;
+            nblk = 0;
             issued = j = 0;
             ok = true;
         }
@@ -903,8 +1046,17 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         // (byte offset >> 4) for buffers and k-steps
         const uint64_t dq0 = sdesc(sbase + Lt::kQOff, 16, 1024);
         const uint64_t dk0 = sdesc(k_src(0, 0), 16, 1024);
+        // (kQSplit) e4m3 operands: query parts hi / lo of buffer b at
+        // kQ8Off + (2 b + part) kQ8Bytes, prefix keys in the stage, block keys (bf16)
+        const uint32_t id_s8 = idesc_e4m3(kRows, kTileKeys);
+        const uint64_t dq8 = sdesc(sbase + Lt::kQ8Off, 16, 1024);
+        const uint64_t dk8 = sdesc(sbase + Lt::kStagesOff, 16, 1024);
+        const uint64_t dkb = sdesc(sbase + Lt::kBlkKOff, 16, 1024);
         const uint64_t dv0 = sdesc(v_src(0, 0), 8192, 1024);
         const uint64_t dp0 = sdesc(sbase + Lt::kPOff, 16, 1024);
+        // rounded row sums: D[64][8] += P[64][64] ones[8][64]^T, column 0 = sum of P
+        const uint64_t d1 = sdesc(sbase + Lt::kOnesOff, 16, 1024);
+        const uint32_t id_l = idesc(kRows, 8, 0, 0);
         bool ok = true;
         if (warp == kSWarp) {
             Walk wsn = w0;
@@ -915,10 +1067,15 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                     qcur = qseg & 1;
                     ok = ok && wait(b_qfull + 8 * qcur, (uint32_t)((qseg >> 1) & 1), abort_flag,
                                     p.status);
+                    // (kQSplit) and split into its e4m3 parts
+                    if (kQSplit)
+                        ok = ok && wait(b_qsplit + 8 * qcur, (uint32_t)((qseg >> 1) & 1),
+                                        abort_flag, p.status);
                 }
                 const int s = (int)(kn % kStages);
-                // the tile's K and V in bf16: landed, and widened if stored as e4m3
-                if (Lt::kConv)
+                // the tile's K and V: landed, and widened if stored as e4m3 (kQSplit:
+                // the e4m3 keys are read as they are)
+                if (Lt::kConv && !kQSplit)
                     ok = ok && wait(b_cready + 8 * (int)(kn % kSlots),
                                     (uint32_t)((kn / kSlots) & 1), abort_flag, p.status);
                 else
@@ -929,21 +1086,41 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                                     (uint32_t)(((kn - kSBufs) / kSBufs) & 1), abort_flag,
                                     p.status);
                 if (!ok) break;
-                const bool seg_end = (wsn.t == wsn.nt - 1) || (kn + 1 == ntiles);
+                const bool blk_tile = wsn.t == wsn.nt - 1;
+                const bool seg_end = blk_tile || (kn + 1 == ntiles);
                 fence_after();
                 if (elect_one()) {
-                    const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
-                    const uint64_t b0 = dk0 + (uint64_t)((k_src(s, kn) - k_src(0, 0)) >> 4);
                     const uint32_t dS = tmem + (uint32_t)((kn % kSBufs) * kTileKeys);
+                    if (kQSplit && !blk_tile) {
+                        // S = hi K^T + lo K^T: 2 x 4 MMAs of 32 e4m3 elements (32 bytes)
+                        const uint64_t ah = dq8 + (uint64_t)((2 * qcur * Lt::kQ8Bytes) >> 4);
+                        const uint64_t al = ah + (uint64_t)(Lt::kQ8Bytes >> 4);
+                        const uint64_t b0 = dk8 + (uint64_t)((s * Lt::kStageBytes) >> 4);
 #pragma unroll
-                    for (int kk = 0; kk < D / 16; ++kk) {
-                        // panel kk / 4, then 16 elements (32 bytes) within the 128-byte row
-                        const uint32_t qoff = ((kk >> 2) * (kRows * 128) + (kk & 3) * 32) >> 4;
-                        const uint32_t koff = ((kk >> 2) * 8192 + (kk & 3) * 32) >> 4;
-                        mma(dS, a0 + qoff, b0 + koff, id_s, kk > 0);
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_e4m3(dS, ah + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), id_s8,
+                                     kk > 0);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_e4m3(dS, al + (uint64_t)(kk * 2), b0 + (uint64_t)(kk * 2), id_s8,
+                                     1u);
+                    } else {
+                        const uint64_t a0 = dq0 + (uint64_t)((qcur * Lt::kQBytes) >> 4);
+                        const uint64_t b0 =
+                            kQSplit ? dkb
+                                    : dk0 + (uint64_t)((k_src(s, kn) - k_src(0, 0)) >> 4);
+#pragma unroll
+                        for (int kk = 0; kk < D / 16; ++kk) {
+                            // panel kk / 4, then 16 elements (32 bytes) within the 128-byte row
+                            const uint32_t qoff =
+                                ((kk >> 2) * (kRows * 128) + (kk & 3) * 32) >> 4;
+                            const uint32_t koff = ((kk >> 2) * 8192 + (kk & 3) * 32) >> 4;
+                            mma(dS, a0 + qoff, b0 + koff, id_s, kk > 0);
+                        }
                     }
                     mma_commit(b_sready + 8 * (int)(kn % kSBufs));
-                    if (KF8) mma_commit(b_kfree + 8 * (int)(kn % kSlots));
+                    if (KF8 && !kQSplit) mma_commit(b_kfree + 8 * (int)(kn % kSlots));
+                    if (kQSplit && blk_tile) mma_commit(b_bkfree);
                     if (seg_end) mma_commit(b_qempty + 8 * qcur);
                 }
                 __syncwarp();
@@ -967,6 +1144,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                         mma(dO, a0 + (uint64_t)((kk * 32) >> 4),
                             b0 + (uint64_t)((kk * 2048) >> 4), id_pv,
                             (!first || kk > 0) ? 1u : 0u);
+#pragma unroll
+                    for (int kk = 0; kk < kTileKeys / 16; ++kk)
+                        mma(dO + D, a0 + (uint64_t)((kk * 32) >> 4), d1 + (uint64_t)((kk * 32) >> 4),
+                            id_l, (!first || kk > 0) ? 1u : 0u);
                     mma_commit(b_pvdone + 8 * (int)(k & 1));
                     mma_commit(b_empty + 8 * s);
                     if (VF8) mma_commit(b_vfree + 8 * (int)(k % kSlots));
@@ -982,6 +1163,31 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         __syncwarp();
         const unsigned long long t0 = globaltimer();
         while (!mbar_try_wait(drain, 0) && globaltimer() - t0 < kWaitNs) {
+        }
+    } else if (kQSplit && warp >= kConvWarp0) {
+        // ========================== query split (kQSplit) ========================
+        // Once a segment's bf16 query rows have landed, split them into their
+        // e4m3 parts for the S MMAs and record each row's e for the softmax
+        // warps (qsplit).  Query buffer b is loaded again only after the S of
+        // its segment and every softmax warp's read of e are done (qempty),
+        // so neither the parts nor e are overwritten early.
+        const int ct = threadIdx.x - kConvWarp0 * 32;
+        Walk wc = w0;
+        int qs = -1;
+        for (long long j = 0; j < ntiles; ++j) {
+            if (j == 0 || wc.t == 0) {
+                ++qs;
+                const int qb = qs & 1;
+                if (!wait(b_qfull + 8 * qb, (uint32_t)((qs >> 1) & 1), abort_flag, p.status))
+                    break;
+                const uint32_t q8 = sbase + Lt::kQ8Off + 2 * qb * Lt::kQ8Bytes;
+                split_q(sbase + Lt::kQOff + qb * Lt::kQBytes, q8, q8 + Lt::kQ8Bytes,
+                        qexp + qb * kRows, ct);
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(b_qsplit + 8 * qb);
+            }
+            walk_next(p, wc);
         }
     } else if (Lt::kConv && warp >= kConvWarp0) {
         // ============================ e4m3 -> bf16 ===============================
@@ -1048,14 +1254,19 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         const bool owner = lane < 16;
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         Walk ws = w0;
-        // l_sum: sum of the fp32 weights 2^(s - m), for the lse; l_rnd: sum of
-        // the same weights as rounded to bf16 for the P V product, for the
-        // normalisation, so that O / l_rnd is an exact convex combination of
+        // l_sum: sum of the fp32 weights 2^(s - m), for the lse.  The sum of
+        // the same weights as rounded to bf16 for the P V product, used for
+        // the normalisation so that O / l is an exact convex combination of
         // the values (the rounding of P then moves the output by a fraction
-        // of the values' spread around it, not of the values themselves)
-        float m_ref = -INFINITY, l_sum = 0.f, l_rnd = 0.f;
+        // of the values' spread around it, not of the values themselves), is
+        // accumulated by the tensor core next to O (P times a ones column,
+        // fp32), which takes its tree of adds off the softmax warps.
+        float m_ref = -INFINITY, l_sum = 0.f;
         int rows_active = 0, irow = 0;
         long long seg_first = lo;
+        // (kQSplit) scale of the prefix tiles' scores: S holds 2^e q.k for this row
+        float row_scale = p.scale_log2;
+        int qs = -1;
         for (long long k = 0; k < ntiles; ++k) {
             const bool first = (k == 0) || (ws.t == 0);
             const bool block_tile = ws.t == ws.nt - 1;
@@ -1063,10 +1274,18 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             if (first) {
                 m_ref = -INFINITY;
                 l_sum = 0.f;
-                l_rnd = 0.f;
                 rows_active = p.G * ws.T;
                 irow = row / p.G;
                 seg_first = lo + k;
+                if (kQSplit) {
+                    ++qs;
+                    const int qb = qs & 1;
+                    wait(b_qsplit + 8 * qb, (uint32_t)((qs >> 1) & 1), abort_flag, p.status);
+                    const int e = qexp[qb * kRows + row];
+                    row_scale = p.scale_log2 * __uint_as_float((uint32_t)(127 - e) << 23);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(b_qempty + 8 * qb);
+                }
             }
             const int nvalid = block_tile ? ws.T : min(kTileKeys, ws.P - ws.t * kTileKeys);
             const int s = (int)(k % kStages);
@@ -1080,7 +1299,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             // mask (rows of other lanes are computed but never stored)
             const int lim = !valid_row ? 0 : (block_tile ? min(nvalid, irow + 1) : nvalid);
             const bool full_tile = !block_tile && nvalid == kTileKeys;
-            const float scale = p.scale_log2;
+            const float scale = kQSplit && !block_tile ? row_scale : p.scale_log2;
             // The thread's 32 scores in registers (masked keys -> -inf); the
             // row's tile max decides the reference first: the segment's first
             // tile sets it, a later tile moves it (rescaling O and l) only when
@@ -1121,10 +1340,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                     if (jump) {
                         m_ref = mt;
                         l_sum *= alpha;
-                        l_rnd *= alpha;
                     }
+                    // O and, in the next 32 columns, the rounded row sum
 #pragma unroll 1
-                    for (int c = 0; c < D; c += 32) {
+                    for (int c = 0; c < D + 32; c += 32) {
                         float o[32];
                         const uint32_t ta = tmem + lane_base + (uint32_t)(kSBufs * kTileKeys + c);
                         tmem_ld32(ta, o);
@@ -1180,25 +1399,15 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
-            {  // the row sums are needed only for l: after P has been handed on
-                float t16[16], r16[16];
+            {  // the row sum is needed only for l: after P has been handed on
+                float t16[16];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    t16[j] = v[j] + v[j + 16];
-                    // word e of w holds P of keys 2e (low half) and 2e + 1
-                    const uint32_t a = w[j >> 1], b = w[(j + 16) >> 1];
-                    r16[j] = (j & 1 ? __uint_as_float(a & 0xFFFF0000u) : __uint_as_float(a << 16)) +
-                             (j & 1 ? __uint_as_float(b & 0xFFFF0000u) : __uint_as_float(b << 16));
-                }
+                for (int j = 0; j < 16; ++j) t16[j] = v[j] + v[j + 16];
 #pragma unroll
                 for (int wd = 8; wd > 0; wd >>= 1)
 #pragma unroll
-                    for (int j = 0; j < wd; ++j) {
-                        t16[j] += t16[j + wd];
-                        r16[j] += r16[j + wd];
-                    }
+                    for (int j = 0; j < wd; ++j) t16[j] += t16[j + wd];
                 l_sum += t16[0];
-                l_rnd += r16[0];
             }
 
             // ---- end of segment: O / l and lse ----
@@ -1210,8 +1419,21 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 const int pair = ws.b * p.Hkv + ws.h;
                 const size_t slot = (size_t)pair + blockIdx.x;
                 const bool write = row < rows_active;
-                // the row's sums: this thread's half plus its partner's
+                // the row's sums: this thread's half plus its partner's; the
+                // rounded one from the tensor core (column 0 of the row-sum
+                // accumulator in the low half, column 1, zero, in the high one)
                 const float l_row = l_sum + __shfl_xor_sync(kFull, l_sum, 16);
+                float l_rnd;
+                {
+                    uint32_t r;
+                    asm volatile(
+                        "tcgen05.ld.sync.aligned.16x32bx2.x1.b32 {%0}, [%1], 1;\n"
+                        "tcgen05.wait::ld.sync.aligned;"
+                        : "=r"(r)
+                        : "r"(tmem + lane_base + (uint32_t)(kSBufs * kTileKeys + D))
+                        : "memory");
+                    l_rnd = __uint_as_float(r);
+                }
                 const float l_row_rnd = l_rnd + __shfl_xor_sync(kFull, l_rnd, 16);
                 const float inv = l_row_rnd > 0.f ? 1.f / l_row_rnd : 0.f;
                 const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;

@@ -36,8 +36,28 @@ def every_code(shape, shift):
     return finite[(np.arange(n) * 7 + shift) % finite.size].reshape(shape)
 
 
+def ranged_q(q):
+    """Query rows over a range of magnitudes, exactly in bf16: row (b, i, h)
+    scaled by 2^k, k cycling through -8..3; every third row's odd elements
+    scaled by a further 2^-12 (far below the row's largest element); one row
+    of zeros per sequence."""
+    x = synth.bf16_bits_to_float(q).astype(np.float64)
+    B, T, H, D = x.shape
+    for b in range(B):
+        for i in range(T):
+            for h in range(H):
+                r = (b * T + i) * H + h
+                x[b, i, h] *= 2.0 ** (r % 12 - 8)
+                if r % 3 == 0:
+                    x[b, i, h, 1::2] *= 2.0 ** -12
+        x[b, 0, H - 1] = 0.0
+    bits = (x.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    assert np.array_equal(synth.bf16_bits_to_float(bits), x.astype(np.float32))  # exact
+    return bits
+
+
 def run_f8(wl, kap, nu, layer=1, prefix=None, block=None, poison_tail=False, scale=0.0,
-           all_codes=False, zero_q=False):
+           all_codes=False, zero_q=False, q_fn=None):
     import paper_2609_34538_gb300 as das
     kt, vt, kl, vl = host_f8_cache(wl)
     if all_codes:
@@ -53,6 +73,8 @@ def run_f8(wl, kap, nu, layer=1, prefix=None, block=None, poison_tail=False, sca
     q = wl_mod.gen_q(wl, layer)
     if zero_q:
         q = np.zeros_like(q)
+    if q_fn is not None:
+        q = q_fn(q)
     kb, vb = wl_mod.gen_block_kv(wl, layer)
     ref_o, ref_l = oracle.attention_f8(kt, vt, kl, vl, layer, kap, nu, pl, bl, q, kb, vb,
                                        scale=scale if scale > 0 else None)
@@ -102,6 +124,16 @@ def test_every_e4m3_code_is_widened_exactly():
     run_f8(small(prefix=(1500, 1500)), 2, 6, all_codes=True)
     for kap, nu in [(6, 3), (4, 4), (2, 6)]:
         run_f8(small(prefix=(1500, 1500)), kap, nu, all_codes=True, zero_q=True)
+
+
+def test_query_magnitudes_e4m3_keys():
+    """e4m3 keys with bf16 values at D = 128 are scored by e4m3 products of
+    the query split into two e4m3 parts under a per-row power of two: query
+    rows over 2^-8..2^3, rows with elements 2^-12 of their largest, and zero
+    rows, against the oracle on the bf16 queries."""
+    run_f8(small(), 2, 6, q_fn=ranged_q)
+    run_f8(small(), 2, 6, q_fn=ranged_q, scale=1.0)
+    run_f8(small(head_dim=64), 2, 6, q_fn=ranged_q)
 
 
 def test_split_across_many_ctas_e4m3():
