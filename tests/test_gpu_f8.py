@@ -136,6 +136,21 @@ def test_query_magnitudes_e4m3_keys():
     run_f8(small(head_dim=64), 2, 6, q_fn=ranged_q)
 
 
+@pytest.mark.parametrize("kap,nu", [(2, 6), (3, 3)])
+def test_ragged_batch_past_32_e4m3(kap, nu):
+    """40 sequences of ragged prefixes 0..300 (some empty) and blocks of 0, 1
+    or 8 rows: a CTA's range holds many segments, so both query buffers turn
+    over many times (the split parts and every softmax warp's read of e are
+    released through qempty), consecutive block tiles reuse the bf16 key
+    buffer (bkfree), and the plan is made after the dependency wait (more than
+    32 sequences)."""
+    wl = small(batch=40, layers=1, q_heads=4, kv_heads=2, prefix=(0, 300), block=(0, 1, 8))
+    P, T = wl.prefix_lens(), wl.block_lens()
+    P[::7] = 0  # empty prefixes: pairs of a block tile alone
+    assert (T == 0).any() and (T == 8).any()
+    run_f8(wl, kap, nu, layer=0, prefix=P, block=T)
+
+
 def test_split_across_many_ctas_e4m3():
     run_f8(small(batch=1, kv_heads=1, q_heads=4, prefix=(20000, 20000), block=(16,)), 2, 6)
 
