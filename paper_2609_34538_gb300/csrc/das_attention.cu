@@ -22,7 +22,10 @@
 //   P V issuer (warp 5) and S issuer (warp 6), one elected lane each, each
 //   blocking on its own in-order barriers:
 //       S = Q K^T    tcgen05.mma M=64 N=64 K=D   -> S buffer (k % 4) in TMEM
+//                    (e4m3 keys at D = 128: two e4m3 passes over the query
+//                    rows split exactly into hi + lo, see split_q)
 //       O += P V     tcgen05.mma M=64 N=D K=64   -> O in TMEM
+//       l += P 1     tcgen05.mma M=64 N=8 K=64   -> the rounded row sums
 //     S of tile k is issued once its K has landed (or been widened) and the
 //     softmax warps have read S buffer k % 4, so the tensor core runs up to
 //     four tiles ahead of the softmax.  A stage is refilled once the P V that
@@ -33,12 +36,13 @@
 //     mask and scale them (base 2), keep a reference max m that only moves
 //     when a score exceeds it by more than 2^8 (then O and l are rescaled in
 //     TMEM), write P = 2^(s - m) as bf16 into a 128-byte-swizzled [64 rows]
-//     [64 keys] buffer (the K-major A operand of P V) and accumulate two row
-//     sums: of the fp32 weights (for the lse) and of the weights as rounded to
-//     bf16 (for the normalisation, so that the output is a convex combination
-//     of the values with exactly the weights the tensor core used).  At the
-//     end of a segment they read the O rows from TMEM and write O / l and the
-//     lse (or the partial).
+//     [64 keys] buffer (the K-major A operand of P V) and accumulate the row
+//     sum of the fp32 weights (for the lse).  The sum of the weights as
+//     rounded to bf16 (for the normalisation, so that the output is a convex
+//     combination of the values with exactly the weights the tensor core
+//     used) is the tensor core's, P times a ones column.  At the end of a
+//     segment they read the O rows and that sum from TMEM and write O / l and
+//     the lse (or the partial).
 // The kernel is launched as a programmatic dependent of the previous kernel
 // in the stream: barrier set-up, the tensor-memory allocation, the work plan
 // (from lengths read before the wait, checked again after it) and an L2
