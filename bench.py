@@ -405,7 +405,7 @@ def gpu_arm(args):
         # the other workloads' attention phases, each on its full cache layout
         # (all R depth slabs allocated), and the long one again on a cache
         # compacted to the two slabs it reads (same bytes; layout effect)
-        probes = {n: draft_probe(n, dev, 200, 5, peak)
+        probes = {n: draft_probe(n, dev, 200, 5, peak, unflushed=(n == "decode"))
                   for n in ("long", "decode", "batched", "verify") if n != args.workload}
         probes["long_2slab"] = draft_probe("long", dev, 200, 5, peak, compact=True)
         commit = commit_probe("verify", dev, 200, 5, peak)
@@ -484,13 +484,16 @@ def gpu_arm(args):
         dist.destroy_process_group()
 
 
-def draft_probe(name, dev, steps, warmup, peak, layers=0, compact=False):
+def draft_probe(name, dev, steps, warmup, peak, layers=0, compact=False, unflushed=False):
     """Per-call time of a workload's attention phase, timed like the main one
     (a CUDA graph of its L layer calls, L2 flushed before every replay), on
     the workload's full cache layout: all R depth slabs allocated, the read
     depths (kappa for keys, nu for values; depth R for both in a verify
     workload) holding the generator's values.  compact=True stores only the
-    two slabs the calls read (the same bytes per call in a smaller cache)."""
+    two slabs the calls read (the same bytes per call in a smaller cache).
+    unflushed=True also times the graph replayed back to back without the
+    flush, for a workload whose per-call bytes fit in L2 (decode: 67 MB per
+    call against 129 MB of L2), reported beside the flushed figure."""
     import torch
 
     import paper_2609_34538_gb300 as das
@@ -542,10 +545,26 @@ def draft_probe(name, dev, steps, warmup, peak, layers=0, compact=False):
             e1.record(stream)
     stream.synchronize()
     ms = [e0.elapsed_time(e1) for e0, e1 in ev[warmup:]]
-    if das.workspace_status(ws) != 0:
-        raise SystemExit(f"bench: {name} attention phase reported a device-side error")
     nbytes = wl.prefix_bytes_per_layer() * L
     gbs = nbytes * len(ms) / (sum(ms) / 1e3) / 1e9
+    extra = {}
+    if unflushed:
+        ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(warmup + steps)]
+        for e0, e1 in ev2:
+            with torch.cuda.stream(stream):
+                e0.record(stream)
+                g.replay()
+                e1.record(stream)
+        stream.synchronize()
+        ms2 = [e0.elapsed_time(e1) for e0, e1 in ev2[warmup:]]
+        gbs2 = nbytes * len(ms2) / (sum(ms2) / 1e3) / 1e9
+        extra = {"unflushed": {"per_call_us": round(statistics.mean(ms2) * 1e3 / L, 2),
+                               "gbs": round(gbs2, 1), "pct_of_measured_hbm": round(100 * gbs2 / peak, 1),
+                               "note": "graph replays back to back, L2 not flushed: part of "
+                                       "each call's bytes may come from L2"}}
+    if das.workspace_status(ws) != 0:
+        raise SystemExit(f"bench: {name} attention phase reported a device-side error")
     cache_gb = 2 * K.numel() * K.element_size() / 1e9
     del K, V, cache, flush
     torch.cuda.empty_cache()
@@ -558,7 +577,7 @@ def draft_probe(name, dev, steps, warmup, peak, layers=0, compact=False):
             "pct_of_nominal_8000": round(100 * gbs / 8000.0, 1),
             "draft_tokens_per_s": (None if verify else
                                    round(int(wl.block_lens().sum()) * len(ms) / (sum(ms) / 1e3), 1)),
-            "steps": len(ms)}
+            "steps": len(ms), **extra}
 
 
 def commit_probe(name, dev, steps, warmup, peak, layers=0, calls=4, vocab=0):
