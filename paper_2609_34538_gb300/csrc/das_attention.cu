@@ -43,6 +43,13 @@
 //     used) is the tensor core's, P times a ones column.  At the end of a
 //     segment they read the O rows and that sum from TMEM and write O / l and
 //     the lse (or the partial).
+// Pairs of at most 16 query rows (decode-shaped calls; bf16, D = 128) take
+// the replicated-rows variant (REP): the rows are loaded four times, at MMA
+// rows 0, 16, 32 and 48, and softmax warp w takes only keys [16 w, 16 w + 16)
+// of its copy, 8 scores a thread instead of 32.  The rest of each copy's P
+// row stays zero, so P V and the row-sum MMA accumulate each copy's own keys;
+// each copy is a softmax of its own (reference max, sums, O rows), and the
+// four are combined by log-sum-exp through shared memory at a segment end.
 // The kernel is launched as a programmatic dependent of the previous kernel
 // in the stream: barrier set-up, the tensor-memory allocation, the work plan
 // (from lengths read before the wait, checked again after it) and an L2
@@ -268,6 +275,21 @@ __device__ __forceinline__ void tmem_ld_half32(uint32_t taddr, float (&v)[32]) {
         : "memory");
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+// (Replicated rows) the calling thread's 8 scores: lane t < 16 of the warp
+// reads TMEM lane t, columns [0, 8) from taddr, lane t + 16 the same lane,
+// columns [8, 16).
+__device__ __forceinline__ void tmem_ld_half8(uint32_t taddr, float (&v)[8]) {
+    uint32_t r[8];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8], 8;\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[j]);
 }
 // The O row of the calling thread's half: with M = 64, thread t < 16 of a warp
 // gets TMEM lane t, columns [64 g, 64 g + 32) for g < D / 64, and thread t + 16
@@ -583,8 +605,10 @@ __device__ bool plan(const AttnParams &p, int P0, int T0, long long &lo, long lo
 //     more DRAM requests in flight per SM.  A pair's block tile is bf16: the
 //     conversion warps load its e4m3-stored operands straight into the ring
 //     slot, the producer the others into the stage.
-template <int D, bool KF8, bool VF8>
+template <int D, bool KF8, bool VF8, bool REP = false>
 struct Layout {
+    static_assert(!REP || (!KF8 && !VF8 && D == 128), "replicated rows: bf16, D = 128");
+    static constexpr bool kRep = REP;
     static constexpr bool kQSplit = KF8 && !VF8 && D == 128;
     static constexpr bool kConv = KF8 || VF8;
     // (kQSplit: 4 stages of 24 KB measured faster than 5, e4m3 long 82.0 -> 81.5 us)
@@ -621,7 +645,13 @@ struct Layout {
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kLenOff = kMiscOff + 16;  // lengths read before the dependency wait
     static constexpr int kQeOff = kLenOff + 64 * 4;  // (kQSplit) e of each row, per query buffer
-    static constexpr int kBytes = kQeOff + (kQSplit ? 2 * kRows * 4 : 0) + 1024;  // + alignment slack
+    // (kRep) the segment end's exchange: each copy's O rows [4][16][kXchStride]
+    // (padded by 16 bytes so that consecutive rows start in different bank
+    // groups), then (m, l, rounded l) of each copy's rows [4][16][4]
+    static constexpr int kXchStride = D + 4;
+    static constexpr int kXchOff = (kQeOff + (kQSplit ? 2 * kRows * 4 : 0) + 15) & ~15;
+    static constexpr int kXchBytes = REP ? (4 * 16 * kXchStride + 4 * 16 * 4) * 4 : 0;
+    static constexpr int kBytes = kXchOff + kXchBytes + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
     static_assert(kBytes <= 232448, "shared memory per CTA");
@@ -772,14 +802,22 @@ template <int D, bool KF8, bool VF8>
 constexpr int kRegCap = Layout<D, KF8, VF8>::kQSplit ? 144 : 255;
 
 // KF8 / VF8: prefix keys / values are e4m3 (tm_k / tm_v are 8-bit maps).
-template <int D, bool KF8, bool VF8>
-__global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
+// REP (bf16, D = 128, at most 16 query rows per pair): replicated rows.  The
+// pair's rows are loaded four times, at MMA rows 0, 16, 32 and 48, so that
+// softmax warp w holds copy w of every row and takes only keys [16 w, 16 w +
+// 16) of each tile (8 a thread instead of 32).  The other keys of its P rows
+// stay zero (the P buffers are cleared once), so P V accumulates each copy's
+// own keys, and each copy keeps its own reference max, sums and O rows; at a
+// segment end the four copies are combined by log-sum-exp through shared
+// memory.
+template <int D, bool KF8, bool VF8, bool REP>
+__global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
     __maxnreg__((kRegCap<D, KF8, VF8>)) attn_kernel(const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_kb,
                    const __grid_constant__ CUtensorMap tm_vb,
                    const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
-    using Lt = Layout<D, KF8, VF8>;
+    using Lt = Layout<D, KF8, VF8, REP>;
     constexpr int kStages = Lt::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -884,6 +922,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                      : "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
+    if (REP) {  // both P buffers start (and, outside each copy's keys, stay) zero
+        for (int i = threadIdx.x; i < 2 * Lt::kPBytes / 16; i += Lt::kThreads)
+            asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                             sbase + Lt::kPOff + i * 16),
+                         "r"(0u)
+                         : "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
     if (warp == kProducerWarp && elect_one()) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_k)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_v)) : "memory");
@@ -949,11 +995,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             if (ok && elect_one()) {
                 const uint32_t full = b_qfull + 8 * qb;
                 const uint32_t dst = sbase + Lt::kQOff + qb * Lt::kQBytes;
-                mbar_arrive_expect_tx(full, Lt::kPanels * p.rows_max * 128);
+                constexpr int kCopies = REP ? 4 : 1;  // (REP) at rows 0, 16, 32, 48
+                mbar_arrive_expect_tx(full, kCopies * Lt::kPanels * p.rows_max * 128);
 #pragma unroll
                 for (int dp = 0; dp < Lt::kPanels; ++dp)
-                    tma_4d(dst + dp * (kRows * 128), &tm_q, full, dp * 64, wl.h * p.G, 0,
-                           wl.b);
+#pragma unroll
+                    for (int c = 0; c < kCopies; ++c)
+                        tma_4d(dst + dp * (kRows * 128) + c * (16 * 128), &tm_q, full, dp * 64,
+                               wl.h * p.G, 0, wl.b);
             }
         }
         const int s = (int)(j % kStages);
@@ -1281,7 +1330,12 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
         // thread (warp, lane) handles row 16 warp + lane % 16, keys of its half
         // (lane / 16) of each tile; the epilogue's O rows are read by lanes < 16
         const int row = warp * 16 + (lane & 15);
+        // (REP) MMA row 16 w + r holds copy w of query row r
+        const int qrow = REP ? (lane & 15) : row;
         const int half = lane >> 4;
+        // scores a thread takes per tile, and the first of them
+        constexpr int kVals = REP ? 8 : 32;
+        const int key0 = REP ? 16 * warp + 8 * half : 32 * half;
         const bool owner = lane < 16;
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         Walk ws = w0;
@@ -1306,7 +1360,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 m_ref = -INFINITY;
                 l_sum = 0.f;
                 rows_active = p.G * ws.T;
-                irow = row / p.G;
+                irow = qrow / p.G;
                 seg_first = lo + k;
                 if (kQSplit) {
                     ++qs;
@@ -1324,8 +1378,9 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             const bool ok_s = wait(b_sready + 8 * (int)(k % kSBufs),
                                    (uint32_t)((k / kSBufs) & 1), abort_flag, p.status);
             fence_after();
-            const uint32_t s_addr = tmem + lane_base + (uint32_t)((k % kSBufs) * kTileKeys);
-            const bool valid_row = row < rows_active && ok_s;
+            const uint32_t s_addr = tmem + lane_base + (uint32_t)((k % kSBufs) * kTileKeys) +
+                                    (uint32_t)(REP ? 16 * warp : 0);
+            const bool valid_row = qrow < rows_active && ok_s;
             // keys j < lim are visible to this row; a full prefix tile needs no
             // mask (rows of other lanes are computed but never stored)
             const int lim = !valid_row ? 0 : (block_tile ? min(nvalid, irow + 1) : nvalid);
@@ -1335,16 +1390,18 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             // row's tile max decides the reference first: the segment's first
             // tile sets it, a later tile moves it (rescaling O and l) only when
             // its max is beyond the reference by more than 2^8.
-            float v[32];
-            tmem_ld_half32(s_addr, v);
+            float v[kVals];
+            if constexpr (REP)
+                tmem_ld_half8(s_addr, v);
+            else
+                tmem_ld_half32(s_addr, v);
             // the scores are in registers: S buffer k % kSBufs may take tile k + kSBufs
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_sfree + 8 * (int)(k % kSBufs));
-            const int key0 = half * 32;
             if (!full_tile) {
 #pragma unroll
-                for (int j = 0; j < 32; j += 2) {
+                for (int j = 0; j < kVals; j += 2) {
                     float a, b;
                     mul2(a, b, v[j], v[j + 1], scale, scale);
                     v[j] = key0 + j < lim ? a : -INFINITY;
@@ -1352,7 +1409,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 }
             }
             float mt;
-            {  // three-input maxima: 32 -> 11 -> 4 -> 1
+            if constexpr (REP) {
+                const float m = max3(max3(v[0], v[1], v[2]), max3(v[3], v[4], v[5]), fmaxf(v[6], v[7]));
+                mt = full_tile ? m * scale : m;
+            } else {  // three-input maxima: 32 -> 11 -> 4 -> 1
                 float m11[11];
 #pragma unroll
                 for (int j = 0; j < 10; ++j) m11[j] = max3(v[3 * j], v[3 * j + 1], v[3 * j + 2]);
@@ -1396,17 +1456,17 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             const float mu = m_ref == -INFINITY ? 0.f : m_ref;
             if (full_tile) {
 #pragma unroll
-                for (int j = 0; j < 32; j += 2)
+                for (int j = 0; j < kVals; j += 2)
                     fma2(v[j], v[j + 1], v[j], v[j + 1], scale, scale, -mu, -mu);
             } else {
 #pragma unroll
-                for (int j = 0; j < 32; j += 2) add2(v[j], v[j + 1], v[j], v[j + 1], -mu, -mu);
+                for (int j = 0; j < kVals; j += 2) add2(v[j], v[j + 1], v[j], v[j + 1], -mu, -mu);
             }
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = ex2(v[j]);
-            uint32_t w[16];
+            for (int j = 0; j < kVals; ++j) v[j] = ex2(v[j]);
+            uint32_t w[kVals / 2];
 #pragma unroll
-            for (int e = 0; e < 16; ++e) w[e] = pack_bf16(v[2 * e], v[2 * e + 1]);
+            for (int e = 0; e < kVals / 2; ++e) w[e] = pack_bf16(v[2 * e], v[2 * e + 1]);
             // P buffer (k & 1) is free once P V of tile k-2, its last reader, is done
             // (pvdone[k & 1] completes once per P V of tiles with that parity)
             if (k >= 2) wait(b_pvdone + 8 * (int)(k & 1), (uint32_t)(((k - 2) >> 1) & 1), abort_flag,
@@ -1414,7 +1474,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             fence_after();
             const uint32_t pbuf = sbase + Lt::kPOff + (uint32_t)((k & 1) * Lt::kPBytes);
 #pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4)
+            for (int q4 = 0; q4 < kVals / 8; ++q4)
                 asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
                                  p_chunk_addr(pbuf, row, key0 / 8 + q4)),
                              "r"(w[4 * q4]), "r"(w[4 * q4 + 1]), "r"(w[4 * q4 + 2]),
@@ -1438,7 +1498,9 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
-            {  // the row sum is needed only for l: after P has been handed on
+            if constexpr (REP) {
+                l_sum += ((v[0] + v[1]) + (v[2] + v[3])) + ((v[4] + v[5]) + (v[6] + v[7]));
+            } else {  // the row sum is needed only for l: after P has been handed on
                 // (packed adds, in the order of the tree t[j] += t[j + w])
                 float t[16];
 #pragma unroll
@@ -1460,7 +1522,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                 const bool whole = (seg_first == pair_first) && block_tile;
                 const int pair = ws.b * p.Hkv + ws.h;
                 const size_t slot = (size_t)pair + blockIdx.x;
-                const bool write = row < rows_active;
+                const bool write = qrow < rows_active;
                 // the row's sums: this thread's half plus its partner's; the
                 // rounded one from the tensor core (column 0 of the row-sum
                 // accumulator in the low half, column 1, zero, in the high one)
@@ -1477,12 +1539,91 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                     l_rnd = __uint_as_float(r);
                 }
                 const float l_row_rnd = l_rnd + __shfl_xor_sync(kFull, l_rnd, 16);
-                const float inv = l_row_rnd > 0.f ? 1.f / l_row_rnd : 0.f;
-                const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;
-                const int gq = row % p.G;
+                const int gq = qrow % p.G;
                 // this thread's columns: [64 g + 32 half, +32) for each 64-column group g
                 float v[D / 2];
                 tmem_ld_orow<D>(tmem + lane_base + (uint32_t)(kSBufs * kTileKeys), v);
+                if constexpr (REP) {
+                    // The four copies of each row through shared memory: every
+                    // copy's O row (not normalised) and its (m, l, rounded l);
+                    // then thread (w, r, half) combines dims [16 (2 w + half),
+                    // +16) of query row r by log-sum-exp over the copies.
+                    float *xo = reinterpret_cast<float *>(sm + Lt::kXchOff);
+                    float *xm = xo + 4 * 16 * Lt::kXchStride;
+                    float *dst = xo + row * Lt::kXchStride + 32 * half;
+#pragma unroll
+                    for (int g = 0; g < D / 64; ++g)
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4)
+                            *reinterpret_cast<float4 *>(dst + 64 * g + j) =
+                                make_float4(v[32 * g + j], v[32 * g + j + 1], v[32 * g + j + 2],
+                                            v[32 * g + j + 3]);
+                    if (half == 0)
+                        *reinterpret_cast<float4 *>(xm + row * 4) =
+                            make_float4(m_ref, l_row, l_row_rnd, 0.f);
+                    asm volatile("bar.sync 1, 128;" ::: "memory");
+                    const int d0 = 16 * (2 * warp + half);
+                    float4 ml[4];
+                    float M = -INFINITY;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        ml[c] = *reinterpret_cast<const float4 *>(xm + (16 * c + qrow) * 4);
+                        M = fmaxf(M, ml[c].x);
+                    }
+                    float L = 0.f, Lr = 0.f, o[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) o[j] = 0.f;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        // a copy that saw no visible key has m = -inf and weight 0
+                        const float sc = ml[c].x == -INFINITY ? 0.f : ex2(ml[c].x - M);
+                        L += sc * ml[c].y;
+                        Lr += sc * ml[c].z;
+                        const float *src = xo + (16 * c + qrow) * Lt::kXchStride + d0;
+#pragma unroll
+                        for (int j = 0; j < 16; j += 4) {
+                            const float4 x = *reinterpret_cast<const float4 *>(src + j);
+                            o[j] += sc * x.x;
+                            o[j + 1] += sc * x.y;
+                            o[j + 2] += sc * x.z;
+                            o[j + 3] += sc * x.w;
+                        }
+                    }
+                    const float inv = Lr > 0.f ? 1.f / Lr : 0.f;
+                    const float lse = L > 0.f ? (M + __log2f(L)) * kLn2 : -INFINITY;
+                    if (write) {
+                        if (whole) {
+                            uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
+                                                      (size_t)ws.h * p.G + gq) * D + d0;
+#pragma unroll
+                            for (int j = 0; j < 16; j += 8)
+                                *reinterpret_cast<uint4 *>(orow + j) =
+                                    make_uint4(pack_bf16(o[j] * inv, o[j + 1] * inv),
+                                               pack_bf16(o[j + 2] * inv, o[j + 3] * inv),
+                                               pack_bf16(o[j + 4] * inv, o[j + 5] * inv),
+                                               pack_bf16(o[j + 6] * inv, o[j + 7] * inv));
+                        } else {
+                            float *prow = p.part_o + (slot * p.rows_max + qrow) * D + d0;
+#pragma unroll
+                            for (int j = 0; j < 16; j += 4)
+                                *reinterpret_cast<float4 *>(prow + j) =
+                                    make_float4(o[j] * inv, o[j + 1] * inv, o[j + 2] * inv,
+                                                o[j + 3] * inv);
+                        }
+                        if (warp == 0 && half == 0) {
+                            if (whole)
+                                p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gq) *
+                                          p.max_block +
+                                      irow] = lse;
+                            else
+                                p.part_lse[slot * p.rows_max + qrow] = lse;
+                        }
+                    }
+                    // the exchange area is free again once every thread has read it
+                    asm volatile("bar.sync 1, 128;" ::: "memory");
+                } else {
+                const float inv = l_row_rnd > 0.f ? 1.f / l_row_rnd : 0.f;
+                const float lse = l_row > 0.f ? (m_ref + __log2f(l_row)) * kLn2 : -INFINITY;
                 if (write) {
                     uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
                                               (size_t)ws.h * p.G + gq) * D + 32 * half;
@@ -1514,6 +1655,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8>::kThreads, 1)
                     else
                         p.part_lse[slot * p.rows_max + row] = lse;
                 }
+                }  // REP
                 if (whole) {  // rows past the block: 0 and lse -inf
                     for (int idx = threadIdx.x; idx < (p.rows_max - rows_active) * (D / 8);
                          idx += kSoftWarps * 32) {
@@ -1733,18 +1875,18 @@ cudaError_t merge_occupancy(int dev, int occ[kMergeVariants]) {
     return cudaSuccess;
 }
 
-template <int D, bool KF8, bool VF8>
+template <int D, bool KF8, bool VF8, bool REP = false>
 cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
                      const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
                      cudaStream_t stream) {
-    using Lt = Layout<D, KF8, VF8>;
+    using Lt = Layout<D, KF8, VF8, REP>;
     constexpr int smem = Lt::kBytes;
     static std::atomic<bool> configured[64];  // the smem opt-in, once per device
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
-        e = cudaFuncSetAttribute(attn_kernel<D, KF8, VF8>,
+        e = cudaFuncSetAttribute(attn_kernel<D, KF8, VF8, REP>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         if (dev < 64) configured[dev].store(true, std::memory_order_release);
@@ -1759,7 +1901,7 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8>, tk, tv, tkb, tvb, tq, p);
+    e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8, REP>, tk, tv, tkb, tvb, tq, p);
     if (e != cudaSuccess) return e;
     // The merge variant with the fewest estimated sequential steps: waves of
     // resident merge CTAs (at least one) times L2 round trips per row (at
@@ -1839,7 +1981,11 @@ cudaError_t attn_launch(const AttnParams &p, int head_dim, bool keys_e4m3, bool 
 #define DAS_LAUNCH(D, K8, V8) tc::launch_d<D, K8, V8>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream)
     if (head_dim == 128) {
         if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(128, true, true) : DAS_LAUNCH(128, true, false);
-        return values_e4m3 ? DAS_LAUNCH(128, false, true) : DAS_LAUNCH(128, false, false);
+        if (values_e4m3) return DAS_LAUNCH(128, false, true);
+        // at most 16 rows per pair: replicated rows (see attn_kernel)
+        return p.rows_max <= 16
+                   ? tc::launch_d<128, false, false, true>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream)
+                   : DAS_LAUNCH(128, false, false);
     }
     if (head_dim == 64) {
         if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(64, true, true) : DAS_LAUNCH(64, true, false);

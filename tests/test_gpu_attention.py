@@ -43,9 +43,11 @@ def test_head_dims(D):
     run_small(small(head_dim=D, q_heads=8, kv_heads=2, prefix=(777, 777), block=(8,)))
 
 
-def test_ragged_batch_with_empty_rows():
-    """Mixed prefix and block lengths, including P = 0 and T = 0."""
-    wl = small(batch=6, q_heads=8, kv_heads=2, block=(16,), prefix=(0, 600))
+@pytest.mark.parametrize("q_heads", [8, 2])
+def test_ragged_batch_with_empty_rows(q_heads):
+    """Mixed prefix and block lengths, including P = 0 and T = 0; 64 and 16
+    rows per kv head at the longest block."""
+    wl = small(batch=6, q_heads=q_heads, kv_heads=2, block=(16,), prefix=(0, 600))
     run_small(wl, prefix=[0, 1, 600, 64, 333, 0], block=[16, 0, 3, 8, 1, 0])
 
 
@@ -118,9 +120,11 @@ def test_one_workspace_across_shapes():
             assert das.workspace_status(ws) == 0
 
 
-def test_sharp_softmax_scale():
-    """scale = 1 makes the softmax peaked (the default 1/sqrt(D) is nearly flat here)."""
-    run_small(small(q_heads=8, kv_heads=2, prefix=(500, 500), block=(8,)), scale=1.0)
+@pytest.mark.parametrize("q_heads", [8, 2])
+def test_sharp_softmax_scale(q_heads):
+    """scale = 1 makes the softmax peaked (the default 1/sqrt(D) is nearly flat
+    here), so the reference max moves often; 32 and 8 rows per kv head."""
+    run_small(small(q_heads=q_heads, kv_heads=2, prefix=(500, 500), block=(8,)), scale=1.0)
 
 
 @pytest.mark.parametrize("kap,nu", [(2, 8), (2, 2), (8, 2), (8, 8), (5, 3)])
@@ -130,8 +134,10 @@ def test_read_policies(kap, nu):
               value_depth=nu)
 
 
-def test_verify_attention():
-    run_small(small(q_heads=8, kv_heads=2, prefix=(400, 400), block=(16,), key_depth=8),
+@pytest.mark.parametrize("q_heads", [8, 2])
+def test_verify_attention(q_heads):
+    """Full-depth verify over 16 candidates: 64 and 16 rows per kv head."""
+    run_small(small(q_heads=q_heads, kv_heads=2, prefix=(400, 400), block=(16,), key_depth=8),
               key_depth=8, value_depth=8, verify=True)
 
 
