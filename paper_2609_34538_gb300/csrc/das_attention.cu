@@ -43,13 +43,14 @@
 //     used) is the tensor core's, P times a ones column.  At the end of a
 //     segment they read the O rows and that sum from TMEM and write O / l and
 //     the lse (or the partial).
-// Pairs of at most 16 query rows (decode-shaped calls; bf16, D = 128) take
-// the replicated-rows variant (REP): the rows are loaded four times, at MMA
-// rows 0, 16, 32 and 48, and softmax warp w takes only keys [16 w, 16 w + 16)
-// of its copy, 8 scores a thread instead of 32.  The rest of each copy's P
-// row stays zero, so P V and the row-sum MMA accumulate each copy's own keys;
-// each copy is a softmax of its own (reference max, sums, O rows), and the
-// four are combined by log-sum-exp through shared memory at a segment end.
+// Pairs of at most 16 (32) query rows (decode-shaped calls; bf16, D = 128)
+// take the replicated-rows variant: the rows are loaded four (two) times, at
+// MMA rows 0, 16, 32 and 48 (0 and 32), and the softmax warps of copy c take
+// only that copy's quarter (half) of every tile's keys, 8 (16) scores a
+// thread instead of 32.  The rest of each copy's P row stays zero, so P V and
+// the row-sum MMA accumulate each copy's own keys; each copy is a softmax of
+// its own (reference max, sums, O rows), and the copies are combined by
+// log-sum-exp through shared memory at a segment end.
 // The kernel is launched as a programmatic dependent of the previous kernel
 // in the stream: barrier set-up, the tensor-memory allocation, the work plan
 // (from lengths read before the wait, checked again after it) and an L2
@@ -290,6 +291,23 @@ __device__ __forceinline__ void tmem_ld_half8(uint32_t taddr, float (&v)[8]) {
         : "memory");
 #pragma unroll
     for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[j]);
+}
+// (Replicated rows, two copies) the calling thread's 16 scores: lane t < 16
+// reads TMEM lane t, columns [0, 16) from taddr, lane t + 16 the same lane,
+// columns [16, 32).
+__device__ __forceinline__ void tmem_ld_half16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15}, [%16], 16;\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
 }
 // The O row of the calling thread's half: with M = 64, thread t < 16 of a warp
 // gets TMEM lane t, columns [64 g, 64 g + 32) for g < D / 64, and thread t + 16
@@ -605,10 +623,11 @@ __device__ bool plan(const AttnParams &p, int P0, int T0, long long &lo, long lo
 //     more DRAM requests in flight per SM.  A pair's block tile is bf16: the
 //     conversion warps load its e4m3-stored operands straight into the ring
 //     slot, the producer the others into the stage.
-template <int D, bool KF8, bool VF8, bool REP = false>
+template <int D, bool KF8, bool VF8, int NC = 1>
 struct Layout {
+    static constexpr bool REP = NC > 1;  // NC copies of the query rows (1, 2 or 4)
+    static_assert(NC == 1 || NC == 2 || NC == 4, "copies: 1, 2 or 4");
     static_assert(!REP || (!KF8 && !VF8 && D == 128), "replicated rows: bf16, D = 128");
-    static constexpr bool kRep = REP;
     static constexpr bool kQSplit = KF8 && !VF8 && D == 128;
     static constexpr bool kConv = KF8 || VF8;
     // (kQSplit: 4 stages of 24 KB measured faster than 5, e4m3 long 82.0 -> 81.5 us)
@@ -645,12 +664,12 @@ struct Layout {
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kLenOff = kMiscOff + 16;  // lengths read before the dependency wait
     static constexpr int kQeOff = kLenOff + 64 * 4;  // (kQSplit) e of each row, per query buffer
-    // (kRep) the segment end's exchange: each copy's O rows [4][16][kXchStride]
+    // (REP) the segment end's exchange: every copy's O rows [kRows][kXchStride]
     // (padded by 16 bytes so that consecutive rows start in different bank
-    // groups), then (m, l, rounded l) of each copy's rows [4][16][4]
+    // groups), then (m, l, rounded l) of every copy's rows [kRows][4]
     static constexpr int kXchStride = D + 4;
     static constexpr int kXchOff = (kQeOff + (kQSplit ? 2 * kRows * 4 : 0) + 15) & ~15;
-    static constexpr int kXchBytes = REP ? (4 * 16 * kXchStride + 4 * 16 * 4) * 4 : 0;
+    static constexpr int kXchBytes = REP ? (kRows * kXchStride + kRows * 4) * 4 : 0;
     static constexpr int kBytes = kXchOff + kXchBytes + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
@@ -802,22 +821,23 @@ template <int D, bool KF8, bool VF8>
 constexpr int kRegCap = Layout<D, KF8, VF8>::kQSplit ? 144 : 255;
 
 // KF8 / VF8: prefix keys / values are e4m3 (tm_k / tm_v are 8-bit maps).
-// REP (bf16, D = 128, at most 16 query rows per pair): replicated rows.  The
-// pair's rows are loaded four times, at MMA rows 0, 16, 32 and 48, so that
-// softmax warp w holds copy w of every row and takes only keys [16 w, 16 w +
-// 16) of each tile (8 a thread instead of 32).  The other keys of its P rows
-// stay zero (the P buffers are cleared once), so P V accumulates each copy's
-// own keys, and each copy keeps its own reference max, sums and O rows; at a
-// segment end the four copies are combined by log-sum-exp through shared
-// memory.
-template <int D, bool KF8, bool VF8, bool REP>
-__global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
+// NC > 1 (bf16, D = 128, at most 64 / NC query rows per pair): replicated
+// rows.  The pair's rows are loaded NC times, copy c at MMA rows [c 64 / NC,
+// (c + 1) 64 / NC), so that the softmax warps of copy c take only keys
+// [c 64 / NC, (c + 1) 64 / NC) of each tile (32 / NC a thread instead of 32).
+// The other keys of their P rows stay zero (the P buffers are cleared once),
+// so P V accumulates each copy's own keys, and each copy keeps its own
+// reference max, sums and O rows; at a segment end the copies are combined
+// by log-sum-exp through shared memory.
+template <int D, bool KF8, bool VF8, int NC>
+__global__ void __launch_bounds__(Layout<D, KF8, VF8, NC>::kThreads, 1)
     __maxnreg__((kRegCap<D, KF8, VF8>)) attn_kernel(const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_kb,
                    const __grid_constant__ CUtensorMap tm_vb,
                    const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
-    using Lt = Layout<D, KF8, VF8, REP>;
+    using Lt = Layout<D, KF8, VF8, NC>;
+    constexpr bool REP = Lt::REP;
     constexpr int kStages = Lt::kStages;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -995,14 +1015,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
             if (ok && elect_one()) {
                 const uint32_t full = b_qfull + 8 * qb;
                 const uint32_t dst = sbase + Lt::kQOff + qb * Lt::kQBytes;
-                constexpr int kCopies = REP ? 4 : 1;  // (REP) at rows 0, 16, 32, 48
-                mbar_arrive_expect_tx(full, kCopies * Lt::kPanels * p.rows_max * 128);
+                // (NC > 1) copy c at rows c 64 / NC
+                mbar_arrive_expect_tx(full, NC * Lt::kPanels * p.rows_max * 128);
 #pragma unroll
                 for (int dp = 0; dp < Lt::kPanels; ++dp)
 #pragma unroll
-                    for (int c = 0; c < kCopies; ++c)
-                        tma_4d(dst + dp * (kRows * 128) + c * (16 * 128), &tm_q, full, dp * 64,
-                               wl.h * p.G, 0, wl.b);
+                    for (int c = 0; c < NC; ++c)
+                        tma_4d(dst + dp * (kRows * 128) + c * (kRows / NC * 128), &tm_q, full,
+                               dp * 64, wl.h * p.G, 0, wl.b);
             }
         }
         const int s = (int)(j % kStages);
@@ -1330,12 +1350,15 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
         // thread (warp, lane) handles row 16 warp + lane % 16, keys of its half
         // (lane / 16) of each tile; the epilogue's O rows are read by lanes < 16
         const int row = warp * 16 + (lane & 15);
-        // (REP) MMA row 16 w + r holds copy w of query row r
-        const int qrow = REP ? (lane & 15) : row;
+        // (REP) MMA row c 64 / NC + r holds copy c of query row r: warp w
+        // holds rows of copy cp = w / (4 / NC)
+        constexpr int kRowsPerCopy = kRows / NC;
+        const int cp = REP ? warp / (4 / NC) : 0;
+        const int qrow = REP ? row - cp * kRowsPerCopy : row;
         const int half = lane >> 4;
         // scores a thread takes per tile, and the first of them
-        constexpr int kVals = REP ? 8 : 32;
-        const int key0 = REP ? 16 * warp + 8 * half : 32 * half;
+        constexpr int kVals = 32 / NC;
+        const int key0 = cp * (kTileKeys / NC) + kVals * half;
         const bool owner = lane < 16;
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         Walk ws = w0;
@@ -1379,7 +1402,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
                                    (uint32_t)((k / kSBufs) & 1), abort_flag, p.status);
             fence_after();
             const uint32_t s_addr = tmem + lane_base + (uint32_t)((k % kSBufs) * kTileKeys) +
-                                    (uint32_t)(REP ? 16 * warp : 0);
+                                    (uint32_t)(cp * (kTileKeys / NC));
             const bool valid_row = qrow < rows_active && ok_s;
             // keys j < lim are visible to this row; a full prefix tile needs no
             // mask (rows of other lanes are computed but never stored)
@@ -1391,8 +1414,10 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
             // tile sets it, a later tile moves it (rescaling O and l) only when
             // its max is beyond the reference by more than 2^8.
             float v[kVals];
-            if constexpr (REP)
+            if constexpr (kVals == 8)
                 tmem_ld_half8(s_addr, v);
+            else if constexpr (kVals == 16)
+                tmem_ld_half16(s_addr, v);
             else
                 tmem_ld_half32(s_addr, v);
             // the scores are in registers: S buffer k % kSBufs may take tile k + kSBufs
@@ -1409,8 +1434,13 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
                 }
             }
             float mt;
-            if constexpr (REP) {
+            if constexpr (kVals == 8) {
                 const float m = max3(max3(v[0], v[1], v[2]), max3(v[3], v[4], v[5]), fmaxf(v[6], v[7]));
+                mt = full_tile ? m * scale : m;
+            } else if constexpr (kVals == 16) {  // 16 -> 6 -> 2 -> 1
+                const float m = fmaxf(max3(max3(v[0], v[1], v[2]), max3(v[3], v[4], v[5]),
+                                           max3(v[6], v[7], v[8])),
+                                      max3(max3(v[9], v[10], v[11]), max3(v[12], v[13], v[14]), v[15]));
                 mt = full_tile ? m * scale : m;
             } else {  // three-input maxima: 32 -> 11 -> 4 -> 1
                 float m11[11];
@@ -1498,8 +1528,19 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_pready + 8 * (int)(k & 1));
-            if constexpr (REP) {
+            if constexpr (kVals == 8) {
                 l_sum += ((v[0] + v[1]) + (v[2] + v[3])) + ((v[4] + v[5]) + (v[6] + v[7]));
+            } else if constexpr (kVals == 16) {
+                float a0, a1, b0, b1;
+                add2(a0, a1, v[0], v[1], v[8], v[9]);
+                add2(b0, b1, v[2], v[3], v[10], v[11]);
+                float c0, c1, d0, d1;
+                add2(c0, c1, v[4], v[5], v[12], v[13]);
+                add2(d0, d1, v[6], v[7], v[14], v[15]);
+                add2(a0, a1, a0, a1, c0, c1);
+                add2(b0, b1, b0, b1, d0, d1);
+                add2(a0, a1, a0, a1, b0, b1);
+                l_sum += a0 + a1;
             } else {  // the row sum is needed only for l: after P has been handed on
                 // (packed adds, in the order of the tree t[j] += t[j + w])
                 float t[16];
@@ -1544,12 +1585,14 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
                 float v[D / 2];
                 tmem_ld_orow<D>(tmem + lane_base + (uint32_t)(kSBufs * kTileKeys), v);
                 if constexpr (REP) {
-                    // The four copies of each row through shared memory: every
+                    // The NC copies of each row through shared memory: every
                     // copy's O row (not normalised) and its (m, l, rounded l);
-                    // then thread (w, r, half) combines dims [16 (2 w + half),
-                    // +16) of query row r by log-sum-exp over the copies.
+                    // then thread (copy cp, row r, half) combines kDims dims of
+                    // query row r, from kDims (2 cp + half), by log-sum-exp
+                    // over the copies.
+                    constexpr int kDims = kRowsPerCopy * D / 128;
                     float *xo = reinterpret_cast<float *>(sm + Lt::kXchOff);
-                    float *xm = xo + 4 * 16 * Lt::kXchStride;
+                    float *xm = xo + kRows * Lt::kXchStride;
                     float *dst = xo + row * Lt::kXchStride + 32 * half;
 #pragma unroll
                     for (int g = 0; g < D / 64; ++g)
@@ -1562,26 +1605,26 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
                         *reinterpret_cast<float4 *>(xm + row * 4) =
                             make_float4(m_ref, l_row, l_row_rnd, 0.f);
                     asm volatile("bar.sync 1, 128;" ::: "memory");
-                    const int d0 = 16 * (2 * warp + half);
-                    float4 ml[4];
+                    const int d0 = kDims * (2 * cp + half);
+                    float4 ml[NC];
                     float M = -INFINITY;
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        ml[c] = *reinterpret_cast<const float4 *>(xm + (16 * c + qrow) * 4);
+                    for (int c = 0; c < NC; ++c) {
+                        ml[c] = *reinterpret_cast<const float4 *>(xm + (c * kRowsPerCopy + qrow) * 4);
                         M = fmaxf(M, ml[c].x);
                     }
-                    float L = 0.f, Lr = 0.f, o[16];
+                    float L = 0.f, Lr = 0.f, o[kDims];
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) o[j] = 0.f;
+                    for (int j = 0; j < kDims; ++j) o[j] = 0.f;
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
+                    for (int c = 0; c < NC; ++c) {
                         // a copy that saw no visible key has m = -inf and weight 0
                         const float sc = ml[c].x == -INFINITY ? 0.f : ex2(ml[c].x - M);
                         L += sc * ml[c].y;
                         Lr += sc * ml[c].z;
-                        const float *src = xo + (16 * c + qrow) * Lt::kXchStride + d0;
+                        const float *src = xo + (c * kRowsPerCopy + qrow) * Lt::kXchStride + d0;
 #pragma unroll
-                        for (int j = 0; j < 16; j += 4) {
+                        for (int j = 0; j < kDims; j += 4) {
                             const float4 x = *reinterpret_cast<const float4 *>(src + j);
                             o[j] += sc * x.x;
                             o[j + 1] += sc * x.y;
@@ -1596,7 +1639,7 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
                             uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
                                                       (size_t)ws.h * p.G + gq) * D + d0;
 #pragma unroll
-                            for (int j = 0; j < 16; j += 8)
+                            for (int j = 0; j < kDims; j += 8)
                                 *reinterpret_cast<uint4 *>(orow + j) =
                                     make_uint4(pack_bf16(o[j] * inv, o[j + 1] * inv),
                                                pack_bf16(o[j + 2] * inv, o[j + 3] * inv),
@@ -1605,12 +1648,12 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, REP>::kThreads, 1)
                         } else {
                             float *prow = p.part_o + (slot * p.rows_max + qrow) * D + d0;
 #pragma unroll
-                            for (int j = 0; j < 16; j += 4)
+                            for (int j = 0; j < kDims; j += 4)
                                 *reinterpret_cast<float4 *>(prow + j) =
                                     make_float4(o[j] * inv, o[j + 1] * inv, o[j + 2] * inv,
                                                 o[j + 3] * inv);
                         }
-                        if (warp == 0 && half == 0) {
+                        if (cp == 0 && half == 0) {
                             if (whole)
                                 p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gq) *
                                           p.max_block +
@@ -1875,18 +1918,18 @@ cudaError_t merge_occupancy(int dev, int occ[kMergeVariants]) {
     return cudaSuccess;
 }
 
-template <int D, bool KF8, bool VF8, bool REP = false>
+template <int D, bool KF8, bool VF8, int NC = 1>
 cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorMap &tv,
                      const CUtensorMap &tkb, const CUtensorMap &tvb, const CUtensorMap &tq,
                      cudaStream_t stream) {
-    using Lt = Layout<D, KF8, VF8, REP>;
+    using Lt = Layout<D, KF8, VF8, NC>;
     constexpr int smem = Lt::kBytes;
     static std::atomic<bool> configured[64];  // the smem opt-in, once per device
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
-        e = cudaFuncSetAttribute(attn_kernel<D, KF8, VF8, REP>,
+        e = cudaFuncSetAttribute(attn_kernel<D, KF8, VF8, NC>,
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         if (dev < 64) configured[dev].store(true, std::memory_order_release);
@@ -1901,7 +1944,7 @@ cudaError_t launch_d(const AttnParams &p, const CUtensorMap &tk, const CUtensorM
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8, REP>, tk, tv, tkb, tvb, tq, p);
+    e = cudaLaunchKernelEx(&cfg, attn_kernel<D, KF8, VF8, NC>, tk, tv, tkb, tvb, tq, p);
     if (e != cudaSuccess) return e;
     // The merge variant with the fewest estimated sequential steps: waves of
     // resident merge CTAs (at least one) times L2 round trips per row (at
@@ -1982,10 +2025,12 @@ cudaError_t attn_launch(const AttnParams &p, int head_dim, bool keys_e4m3, bool 
     if (head_dim == 128) {
         if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(128, true, true) : DAS_LAUNCH(128, true, false);
         if (values_e4m3) return DAS_LAUNCH(128, false, true);
-        // at most 16 rows per pair: replicated rows (see attn_kernel)
-        return p.rows_max <= 16
-                   ? tc::launch_d<128, false, false, true>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream)
-                   : DAS_LAUNCH(128, false, false);
+        // at most 16 (32) rows per pair: four (two) copies of the rows (see attn_kernel)
+        if (p.rows_max <= 16)
+            return tc::launch_d<128, false, false, 4>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+        if (p.rows_max <= 32)
+            return tc::launch_d<128, false, false, 2>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+        return DAS_LAUNCH(128, false, false);
     }
     if (head_dim == 64) {
         if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(64, true, true) : DAS_LAUNCH(64, true, false);

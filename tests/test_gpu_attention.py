@@ -32,9 +32,10 @@ def test_prefix_lengths(P):
 
 
 @pytest.mark.parametrize("G,T", [(1, 1), (1, 16), (4, 4), (4, 8), (4, 12), (4, 16), (8, 8),
-                                 (1, 64), (2, 32)])
+                                 (1, 64), (2, 32), (1, 17), (2, 16), (1, 32)])
 def test_rows_per_kv_head(G, T):
-    """1..4 m-tiles of 16 rows (keys split 4, 2 or 1 ways between warps)."""
+    """1..64 rows per kv head: up to 16 and up to 32 rows take four and two
+    copies of the rows, more the 64-row layout."""
     run_small(small(q_heads=2 * G, kv_heads=2, prefix=(300, 300), block=(T,)))
 
 
