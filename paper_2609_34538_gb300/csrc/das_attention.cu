@@ -43,8 +43,9 @@
 //     used) is the tensor core's, P times a ones column.  At the end of a
 //     segment they read the O rows and that sum from TMEM and write O / l and
 //     the lse (or the partial).
-// Pairs of at most 16 (32) query rows (decode-shaped calls; bf16, D = 128)
-// take the replicated-rows variant: the rows are loaded four (two) times, at
+// Pairs of at most 16 (32) query rows (decode-shaped calls; D = 128, bf16
+// values, keys bf16 or e4m3 with split-query scores) take the
+// replicated-rows variant: the rows are loaded four (two) times, at
 // MMA rows 0, 16, 32 and 48 (0 and 32), and the softmax warps of copy c take
 // only that copy's quarter (half) of every tile's keys, 8 (16) scores a
 // thread instead of 32.  The rest of each copy's P row stays zero, so P V and
@@ -627,7 +628,8 @@ template <int D, bool KF8, bool VF8, int NC = 1>
 struct Layout {
     static constexpr bool REP = NC > 1;  // NC copies of the query rows (1, 2 or 4)
     static_assert(NC == 1 || NC == 2 || NC == 4, "copies: 1, 2 or 4");
-    static_assert(!REP || (!KF8 && !VF8 && D == 128), "replicated rows: bf16, D = 128");
+    // bf16 keys, or e4m3 keys with the split-query scores; bf16 values; D = 128
+    static_assert(!REP || (!VF8 && D == 128), "replicated rows: bf16 values, D = 128");
     static constexpr bool kQSplit = KF8 && !VF8 && D == 128;
     static constexpr bool kConv = KF8 || VF8;
     // (kQSplit: 4 stages of 24 KB measured faster than 5, e4m3 long 82.0 -> 81.5 us)
@@ -664,12 +666,23 @@ struct Layout {
     static constexpr int kMiscOff = kBarOff + kNumBars * 8;
     static constexpr int kLenOff = kMiscOff + 16;  // lengths read before the dependency wait
     static constexpr int kQeOff = kLenOff + 64 * 4;  // (kQSplit) e of each row, per query buffer
-    // (REP) the segment end's exchange: every copy's O rows [kRows][kXchStride]
-    // (padded by 16 bytes so that consecutive rows start in different bank
-    // groups), then (m, l, rounded l) of every copy's rows [kRows][4]
-    static constexpr int kXchStride = D + 4;
+    // (REP) the segment end's exchange, then (m, l, rounded l) of every MMA
+    // row [kRows][4]; rows are padded by 16 bytes so that consecutive rows
+    // start in different bank groups.  Compacted (e4m3 keys, whose stages
+    // leave too little shared memory for whole rows): a softmax thread holds
+    // D / 2 values of its copy's O row, in NC groups of D / 2 / NC; each
+    // group is combined by the thread of the copy with its index, so a thread
+    // stores only the NC - 1 groups other copies combine: [2 halves][kRows]
+    // [kXchStride] floats.
+    // With bf16 keys there is room for the whole rows: every copy's O row
+    // [kRows][kXchStride] (measured faster for bf16: decode 17.43 -> 17.12 us).
+    static constexpr bool kCompactXch = KF8;
+    static constexpr int kXchStride =
+        !REP ? 0 : kCompactXch ? (NC - 1) * (D / 2 / NC) + 4 : D + 4;
     static constexpr int kXchOff = (kQeOff + (kQSplit ? 2 * kRows * 4 : 0) + 15) & ~15;
-    static constexpr int kXchBytes = REP ? (kRows * kXchStride + kRows * 4) * 4 : 0;
+    static constexpr int kXchBytes =
+        !REP ? 0
+             : ((kCompactXch ? 2 * kRows * kXchStride : kRows * kXchStride) + kRows * 4) * 4;
     static constexpr int kBytes = kXchOff + kXchBytes + 1024;  // + alignment slack
     static_assert(kStageBytes % 1024 == 0 && kKBytes % 1024 == 0 && kConvBytes % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
@@ -821,8 +834,8 @@ template <int D, bool KF8, bool VF8>
 constexpr int kRegCap = Layout<D, KF8, VF8>::kQSplit ? 144 : 255;
 
 // KF8 / VF8: prefix keys / values are e4m3 (tm_k / tm_v are 8-bit maps).
-// NC > 1 (bf16, D = 128, at most 64 / NC query rows per pair): replicated
-// rows.  The pair's rows are loaded NC times, copy c at MMA rows [c 64 / NC,
+// NC > 1 (D = 128, bf16 values, at most 64 / NC query rows per pair):
+// replicated rows.  The pair's rows are loaded NC times, copy c at MMA rows [c 64 / NC,
 // (c + 1) 64 / NC), so that the softmax warps of copy c take only keys
 // [c 64 / NC, (c + 1) 64 / NC) of each tile (32 / NC a thread instead of 32).
 // The other keys of their P rows stay zero (the P buffers are cleared once),
@@ -1584,7 +1597,110 @@ __global__ void __launch_bounds__(Layout<D, KF8, VF8, NC>::kThreads, 1)
                 // this thread's columns: [64 g + 32 half, +32) for each 64-column group g
                 float v[D / 2];
                 tmem_ld_orow<D>(tmem + lane_base + (uint32_t)(kSBufs * kTileKeys), v);
-                if constexpr (REP) {
+                if constexpr (REP && Lt::kCompactXch) {
+                    // The NC copies of each row through shared memory: the
+                    // groups of its O row (not normalised) that the other
+                    // copies combine, and its (m, l, rounded l); then thread
+                    // (copy cp, row r, half) combines group cp of half `half`
+                    // of query row r by log-sum-exp over the copies.
+                    constexpr int kG = D / 2 / NC;  // values per group
+                    constexpr int kXS = Lt::kXchStride;
+                    float *xo = reinterpret_cast<float *>(sm + Lt::kXchOff);
+                    float *xm = xo + 2 * kRows * kXS;
+                    float *dst = xo + (half * kRows + row) * kXS;
+#pragma unroll
+                    for (int g = 0; g < NC; ++g) {
+                        if (g == cp) continue;
+                        const int slot = g < cp ? g : g - 1;
+#pragma unroll
+                        for (int j = 0; j < kG; j += 4)
+                            *reinterpret_cast<float4 *>(dst + slot * kG + j) =
+                                make_float4(v[g * kG + j], v[g * kG + j + 1], v[g * kG + j + 2],
+                                            v[g * kG + j + 3]);
+                    }
+                    if (half == 0)
+                        *reinterpret_cast<float4 *>(xm + row * 4) =
+                            make_float4(m_ref, l_row, l_row_rnd, 0.f);
+                    // this thread's own group, selected without a dynamic register index
+                    constexpr int kDims = kG;
+                    float own[kG];
+#pragma unroll
+                    for (int j = 0; j < kG; ++j) own[j] = v[j];
+#pragma unroll
+                    for (int g = 1; g < NC; ++g)
+                        if (cp == g)
+#pragma unroll
+                            for (int j = 0; j < kG; ++j) own[j] = v[g * kG + j];
+                    asm volatile("bar.sync 1, 128;" ::: "memory");
+                    // group cp's dims: values [0, 32) of a half are dims 32 half + i,
+                    // values [32, 64) dims 64 + 32 half + i - 32
+                    const int i0 = cp * kG;
+                    const int d0 = i0 < 32 ? 32 * half + i0 : 64 + 32 * half + (i0 - 32);
+                    float4 ml[NC];
+                    float M = -INFINITY;
+#pragma unroll
+                    for (int c = 0; c < NC; ++c) {
+                        ml[c] = *reinterpret_cast<const float4 *>(xm + (c * kRowsPerCopy + qrow) * 4);
+                        M = fmaxf(M, ml[c].x);
+                    }
+                    float L = 0.f, Lr = 0.f, o[kDims];
+#pragma unroll
+                    for (int j = 0; j < kDims; ++j) o[j] = 0.f;
+#pragma unroll
+                    for (int c = 0; c < NC; ++c) {
+                        // a copy that saw no visible key has m = -inf and weight 0
+                        const float sc = ml[c].x == -INFINITY ? 0.f : ex2(ml[c].x - M);
+                        L += sc * ml[c].y;
+                        Lr += sc * ml[c].z;
+                        if (c == cp) {
+#pragma unroll
+                            for (int j = 0; j < kDims; ++j) o[j] += sc * own[j];
+                        } else {
+                            const float *src = xo + (half * kRows + c * kRowsPerCopy + qrow) * kXS +
+                                               (cp < c ? cp : cp - 1) * kG;
+#pragma unroll
+                            for (int j = 0; j < kDims; j += 4) {
+                                const float4 x = *reinterpret_cast<const float4 *>(src + j);
+                                o[j] += sc * x.x;
+                                o[j + 1] += sc * x.y;
+                                o[j + 2] += sc * x.z;
+                                o[j + 3] += sc * x.w;
+                            }
+                        }
+                    }
+                    const float inv = Lr > 0.f ? 1.f / Lr : 0.f;
+                    const float lse = L > 0.f ? (M + __log2f(L)) * kLn2 : -INFINITY;
+                    if (write) {
+                        if (whole) {
+                            uint16_t *orow = p.out + (((size_t)ws.b * p.max_block + irow) * p.Hq +
+                                                      (size_t)ws.h * p.G + gq) * D + d0;
+#pragma unroll
+                            for (int j = 0; j < kDims; j += 8)
+                                *reinterpret_cast<uint4 *>(orow + j) =
+                                    make_uint4(pack_bf16(o[j] * inv, o[j + 1] * inv),
+                                               pack_bf16(o[j + 2] * inv, o[j + 3] * inv),
+                                               pack_bf16(o[j + 4] * inv, o[j + 5] * inv),
+                                               pack_bf16(o[j + 6] * inv, o[j + 7] * inv));
+                        } else {
+                            float *prow = p.part_o + (slot * p.rows_max + qrow) * D + d0;
+#pragma unroll
+                            for (int j = 0; j < kDims; j += 4)
+                                *reinterpret_cast<float4 *>(prow + j) =
+                                    make_float4(o[j] * inv, o[j + 1] * inv, o[j + 2] * inv,
+                                                o[j + 3] * inv);
+                        }
+                        if (cp == 0 && half == 0) {
+                            if (whole)
+                                p.lse[((size_t)ws.b * p.Hq + (size_t)ws.h * p.G + gq) *
+                                          p.max_block +
+                                      irow] = lse;
+                            else
+                                p.part_lse[slot * p.rows_max + qrow] = lse;
+                        }
+                    }
+                    // the exchange area is free again once every thread has read it
+                    asm volatile("bar.sync 1, 128;" ::: "memory");
+                } else if constexpr (REP) {
                     // The NC copies of each row through shared memory: every
                     // copy's O row (not normalised) and its (m, l, rounded l);
                     // then thread (copy cp, row r, half) combines kDims dims of
@@ -2023,7 +2139,14 @@ cudaError_t attn_launch(const AttnParams &p, int head_dim, bool keys_e4m3, bool 
                         const CUtensorMap &tm_q, cudaStream_t stream) {
 #define DAS_LAUNCH(D, K8, V8) tc::launch_d<D, K8, V8>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream)
     if (head_dim == 128) {
-        if (keys_e4m3) return values_e4m3 ? DAS_LAUNCH(128, true, true) : DAS_LAUNCH(128, true, false);
+        if (keys_e4m3) {
+            if (values_e4m3) return DAS_LAUNCH(128, true, true);
+            if (p.rows_max <= 16)
+                return tc::launch_d<128, true, false, 4>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+            if (p.rows_max <= 32)
+                return tc::launch_d<128, true, false, 2>(p, tm_k, tm_v, tm_kb, tm_vb, tm_q, stream);
+            return DAS_LAUNCH(128, true, false);
+        }
         if (values_e4m3) return DAS_LAUNCH(128, false, true);
         // at most 16 (32) rows per pair: four (two) copies of the rows (see attn_kernel)
         if (p.rows_max <= 16)
